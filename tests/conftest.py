@@ -1,0 +1,91 @@
+import os
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def pytest_configure(config):
+    config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300); runs the replay kernels through the C ABI")
+    config.addinivalue_line("markers", "slow: long-running; selected only when NDVM_SLOW=1")
+
+
+def pytest_collection_modifyitems(config, items):
+    if os.environ.get("NDVM_SLOW") == "1":
+        return
+    skip = pytest.mark.skip(reason="slow test (set NDVM_SLOW=1)")
+    for it in items:
+        if "slow" in it.keywords:
+            it.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def oracle_mod():
+    import oracle
+    oracle.build()
+    return oracle
+
+
+@pytest.fixture(scope="session")
+def ndvm():
+    import paper_2607_03574_gb300 as nd
+    nd.load()
+    return nd
+
+
+@pytest.fixture(scope="session")
+def cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("GPU test selected but no CUDA device is visible")
+    return torch.device("cuda:0")
+
+
+def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol, mag=None):
+    """Comparison rule for one batch of lanes.
+
+    Loss: |gpu - ora| <= tol * |ora|.  Gradient component k: |gpu - ora| <= tol * s_k with
+    s_k = max(max_j |ora gradient_j| of that lane, mag_k), where mag_k (from the oracle's
+    magnitude mode) is the component propagated through absolute values -- the size of
+    the terms it sums.  A component that is a small difference of large terms is thus
+    judged against those terms, the scale any summation order's rounding is bounded by.  A lane whose oracle loss is non-finite must be non-finite
+    in the same class (NaN vs +-inf) on the GPU and is excluded from the relative checks.
+    Returns (ok, report).
+    """
+    gpu_loss = np.asarray(gpu_loss, dtype=np.float64)
+    ora_loss = np.asarray(ora_loss, dtype=np.float64)
+    fin = np.isfinite(ora_loss)
+    bad = []
+    if (~fin).any():
+        for b in np.nonzero(~fin)[0]:
+            same = (np.isnan(ora_loss[b]) and np.isnan(gpu_loss[b])) or (ora_loss[b] == gpu_loss[b])
+            if not same:
+                bad.append(f"lane {b}: non-finite class {ora_loss[b]} vs {gpu_loss[b]}")
+    el = np.abs(gpu_loss[fin] - ora_loss[fin]) / np.maximum(np.abs(ora_loss[fin]), 1e-300)
+    worst_l = float(el.max()) if el.size else 0.0
+    if worst_l > tol:
+        b = np.nonzero(fin)[0][int(np.argmax(el))]
+        bad.append(f"loss lane {b}: gpu {gpu_loss[b]!r} oracle {ora_loss[b]!r} rel {worst_l:.3e}")
+    worst_g = 0.0
+    if gpu_grad is not None and ora_grad is not None and ora_grad.size:
+        g = np.asarray(gpu_grad, dtype=np.float64)[fin]
+        o = np.asarray(ora_grad, dtype=np.float64)[fin]
+        gfin = np.isfinite(o).all(axis=1)
+        s = np.max(np.abs(o[gfin]), axis=1, keepdims=True)
+        if mag is not None:
+            s = np.maximum(s, np.asarray(mag, dtype=np.float64)[fin][gfin])
+        s = np.maximum(s, 1e-300)
+        eg = np.abs(g[gfin] - o[gfin]) / s
+        worst_g = float(eg.max()) if eg.size else 0.0
+        if worst_g > tol:
+            i, k = np.unravel_index(int(np.argmax(eg)), eg.shape)
+            bad.append(f"grad lane {i} comp {k}: gpu {g[gfin][i, k]!r} oracle {o[gfin][i, k]!r} rel {worst_g:.3e}")
+        nf = ~gfin
+        if nf.any() and not np.array_equal(np.isnan(g[nf]), np.isnan(o[nf])):
+            bad.append("non-finite gradient class mismatch")
+    return (not bad), {"worst_loss": worst_l, "worst_grad": worst_g, "nonfinite_lanes": int((~fin).sum()),
+                       "problems": bad}

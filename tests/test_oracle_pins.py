@@ -1,0 +1,424 @@
+"""Pins of the oracle to things other than itself (no GPU).
+
+Each test checks the oracle's loss and gradient against an independent fact:
+closed-form gradients, the dense-Gaussian form of a Kalman likelihood, a
+forward-sensitivity recursion, central finite differences, and invariants.  The
+reverse mode and the dual-number mode of the oracle are also checked against each
+other on every workload.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import workloads as W
+
+REV, DUAL, VAL = 0 + 1, 2, 0
+
+
+def run(oracle_mod, prog, params, obs=(), frontend=0, mode=1):
+    return oracle_mod.run(prog, np.atleast_2d(np.asarray(params, dtype=float)), np.asarray(obs, dtype=float),
+                          frontend=frontend, mode=mode)
+
+
+def assert_rel(a, b, tol, scale=None):
+    a, b = np.asarray(a, float), np.asarray(b, float)
+    s = np.maximum(np.abs(b), 1e-300) if scale is None else scale
+    err = np.max(np.abs(a - b) / s)
+    assert err <= tol, (err, a, b)
+
+
+# ---------------------------------------------------------------- closed forms
+LINREG = """
+(model (params a b)
+  (/ (data-sum {n} 2 (let ((r (- (+ (* a (dobs 0)) b) (dobs 1)))) (* r r))) {nf}))
+"""
+
+
+def test_linear_regression_closed_form(oracle_mod):
+    rng = np.random.default_rng(11)
+    n = 40
+    x = rng.uniform(-3, 3, n)
+    y = 0.7 * x - 1.2 + rng.normal(0, 0.3, n)
+    obs = np.stack([x, y], 1).reshape(-1)
+    th = rng.normal(0, 1, (6, 2))
+    loss, grad = run(oracle_mod, LINREG.format(n=n, nf=f"{n}.0"), th, obs)
+    for b in range(6):
+        r = th[b, 0] * x + th[b, 1] - y
+        assert_rel(loss[b], np.mean(r * r), 1e-13)
+        assert_rel(grad[b], [2 * np.mean(r * x), 2 * np.mean(r)], 1e-12, scale=np.max(np.abs(grad[b])))
+
+
+def test_exp_decay_closed_form(oracle_mod):
+    w = W.exp_decay(B=16)
+    loss, grad = run(oracle_mod, w.program, w.params, w.obs)
+    t, y = w.obs[0::2], w.obs[1::2]
+    for b in range(w.B):
+        a, k, c = w.params[b]
+        e = np.exp(-k * t)
+        r = a * e + c - y
+        assert_rel(loss[b], np.mean(r * r), 1e-13)
+        g = [2 * np.mean(r * e), -2 * np.mean(r * a * t * e), 2 * np.mean(r)]
+        assert_rel(grad[b], g, 1e-12, scale=np.max(np.abs(g)))
+
+
+# ---------------------------------------------- Kalman: dense Gaussian identity
+SCALAR_KALMAN = """
+(define (nll q r y0 T)
+  (let loop ((t 0) (x 0.0) (P {p0}) (acc 0.0))
+    (if (= t T) acc
+        (let* ((Pp (+ P q)) (S (+ Pp r)) (v (- (obs t) x)) (K (/ Pp S)))
+          (loop (+ t 1) (+ x (* K v)) (* (- 1.0 K) Pp)
+                (+ acc (* 0.5 (+ (log S) (/ (* v v) S) 1.8378770664093453))))))))
+(model (params lq lr) (nll (exp lq) (exp lr) 0 {T}))
+"""
+
+
+def dense_gaussian_nll(y, Sig, dSig):
+    """NLL of y ~ N(0, Sig) and its gradient given dSig/dtheta_k (list)."""
+    L = np.linalg.cholesky(Sig)
+    alpha = np.linalg.solve(Sig, y)
+    nll = 0.5 * (2 * np.sum(np.log(np.diag(L))) + y @ alpha + len(y) * math.log(2 * math.pi))
+    Si = np.linalg.inv(Sig)
+    g = [0.5 * np.trace(Si @ D) - 0.5 * alpha @ D @ alpha for D in dSig]
+    return nll, np.array(g)
+
+
+def test_scalar_random_walk_kalman_is_dense_gaussian(oracle_mod):
+    rng = np.random.default_rng(3)
+    T, p0 = 30, 2.5
+    y = np.cumsum(rng.normal(0, 0.5, T)) + rng.normal(0, 0.4, T)
+    th = np.array([[math.log(0.25), math.log(0.16)], [math.log(1.3), math.log(0.02)], [0.1, -0.3]])
+    loss, grad = run(oracle_mod, SCALAR_KALMAN.format(p0=repr(p0), T=T), th, y)
+    i = np.arange(1, T + 1)
+    Lm = np.minimum.outer(i, i).astype(float)
+    for b in range(len(th)):
+        q, r = np.exp(th[b])
+        Sig = p0 + q * Lm + r * np.eye(T)
+        nll, g = dense_gaussian_nll(y, Sig, [q * Lm, r * np.eye(T)])
+        assert_rel(loss[b], nll, 1e-11)
+        assert_rel(grad[b], g, 1e-10, scale=np.max(np.abs(g)))
+
+
+def lgssm_dense_cov(F, H, Q, R, P0, T):
+    """Covariance of the stacked observations of x_t = F x_{t-1} + w_t, y_t = H x_t + v_t, x_0 ~ N(0, P0)."""
+    n, m = F.shape[0], H.shape[0]
+    cov = [None] * (T + 1)
+    cov[0] = P0
+    for t in range(1, T + 1):
+        cov[t] = F @ cov[t - 1] @ F.T + Q
+    Sig = np.zeros((m * T, m * T))
+    for t in range(1, T + 1):
+        for s in range(1, t + 1):
+            Ft = np.linalg.matrix_power(F, t - s)
+            C = H @ Ft @ cov[s] @ H.T
+            Sig[(t - 1) * m:t * m, (s - 1) * m:s * m] = C
+            Sig[(s - 1) * m:s * m, (t - 1) * m:t * m] = C.T
+        Sig[(t - 1) * m:t * m, (t - 1) * m:t * m] += R
+    return Sig
+
+
+def test_kalman_cv4_is_dense_gaussian(oracle_mod):
+    T = 6
+    w = W.kalman_cv4(B=5, T=T)
+    loss, grad = run(oracle_mod, w.program, w.params, w.obs[: 2 * T])
+    F = np.array([[1, 0, 1, 0], [0, 1, 0, 1], [0, 0, 1, 0], [0, 0, 0, 1]], float)
+    H = np.eye(2, 4)
+    P0 = 10 * np.eye(4)
+
+    def sig(v):
+        qx, qy, rx, ry = v
+        Q = np.array([[qx / 3, 0, qx / 2, 0], [0, qy / 3, 0, qy / 2], [qx / 2, 0, qx, 0], [0, qy / 2, 0, qy]])
+        return lgssm_dense_cov(F, H, Q, np.diag([rx, ry]), P0, T)
+
+    base = sig(np.zeros(4))
+    A = [sig(np.eye(4)[k]) - base for k in range(4)]   # Sigma is affine in the variances
+    y = w.obs[: 2 * T]
+    for b in range(w.B):
+        v = np.exp(2 * w.params[b])
+        Sig = base + sum(v[k] * A[k] for k in range(4))
+        nll, g = dense_gaussian_nll(y, Sig, [2 * v[k] * A[k] for k in range(4)])
+        assert_rel(loss[b], nll, 1e-11)
+        assert_rel(grad[b], g, 1e-9, scale=np.max(np.abs(g)))
+
+
+def test_kalman_rand8_is_dense_gaussian(oracle_mod):
+    T = 4
+    w = W.kalman_rand8(B=3, T=T)
+    F = w.meta["F"]
+    n, m = 8, 3
+    H = np.zeros((m, n))
+    H[:, :m] = np.eye(m)
+    y = w.obs[: m * T]
+    loss, grad = run(oracle_mod, w.program, w.params, y)
+
+    def sig(v):
+        return lgssm_dense_cov(F, H, np.diag(v[:n]), np.diag(v[n:n + m]), v[-1] * np.eye(n), T)
+
+    base = sig(np.zeros(n + m + 1))
+    A = [sig(np.eye(n + m + 1)[k]) - base for k in range(n + m + 1)]
+    for b in range(w.B):
+        v = np.exp(2 * w.params[b])
+        Sig = base + sum(v[k] * A[k] for k in range(n + m + 1))
+        nll, g = dense_gaussian_nll(y, Sig, [2 * v[k] * A[k] for k in range(n + m + 1)])
+        assert_rel(loss[b], nll, 1e-10)
+        assert_rel(grad[b], g, 1e-8, scale=np.max(np.abs(g)))
+
+
+# --------------------------------------------------- logistic: tangent-linear recursion
+def test_logistic_forward_sensitivity(oracle_mod):
+    w = W.logistic(B=6)
+    loss, grad = run(oracle_mod, w.program, w.params, w.obs, frontend=1)
+    dt = 0.01
+    for b in range(w.B):
+        r, K = w.params[b]
+        x, s = 0.1, np.zeros(2)
+        se, gacc = 0.0, np.zeros(2)
+        k = 0
+        for n in range(1000):
+            f_x = r * (1 - 2 * x / K)
+            f_th = np.array([x * (1 - x / K), r * x * x / (K * K)])
+            s = s + dt * (f_x * s + f_th)
+            x = x + dt * (r * x * (1 - x / K))
+            if (n + 1) % 10 == 0:
+                res = x - w.obs[k]
+                se += res * res
+                gacc += 2 * res * s
+                k += 1
+        assert_rel(loss[b], se / 100, 1e-12)
+        assert_rel(grad[b], gacc / 100, 1e-11, scale=np.max(np.abs(gacc / 100)))
+
+
+# ---------------------------------------------------------- finite differences
+def central_fd(oracle_mod, prog, th, obs, frontend=0):
+    th = np.asarray(th, float)
+    P = th.size
+    rows = []
+    hs = 1e-5 * np.maximum(1.0, np.abs(th))
+    for k in range(P):
+        for sgn in (1, -1):
+            t = th.copy()
+            t[k] += sgn * hs[k]
+            rows.append(t)
+    lv, _ = run(oracle_mod, prog, np.array(rows), obs, frontend=frontend, mode=0)
+    return (lv[0::2] - lv[1::2]) / (2 * hs)
+
+
+@pytest.mark.parametrize("i", range(12))
+def test_random_programs_match_finite_differences(oracle_mod, i):
+    w = W.random_exprs(n_programs=12, B=2, n_points=24, seed=99)[i]
+    loss, grad = run(oracle_mod, w.program, w.params, w.obs)
+    for b in range(w.B):
+        fd = central_fd(oracle_mod, w.program, w.params[b], w.obs)
+        assert_rel(grad[b], fd, 2e-6, scale=max(np.max(np.abs(grad[b])), 1e-3))
+
+
+def test_kalman_matches_finite_differences(oracle_mod):
+    w = W.kalman_cv4(B=2, T=25)
+    _, grad = run(oracle_mod, w.program, w.params, w.obs)
+    for b in range(w.B):
+        fd = central_fd(oracle_mod, w.program, w.params[b], w.obs)
+        assert_rel(grad[b], fd, 1e-6, scale=np.max(np.abs(grad[b])))
+
+
+# -------------------------------------------------- matrix primitives (App. C)
+MATPROG = """
+(model (params a b c d e f g h i)
+  (let* ((A (matrix 3 3 a b c d e f g h i))
+         (S (m+ (matmul A (transpose A)) (identity 3)))
+         (B2 (submatrix A 0 2 1 2)))
+    (+ (det A) (logdet S) (trace (matmul (inv S) A)) (mref (inv B2) 0 1)
+       (* 0.5 (dot (matmul A (matrix 3 1 1.0 -2.0 0.5)) (matrix 3 1 0.3 0.2 0.1)))
+       (trace (mscale a A)))))
+"""
+
+
+def test_matrix_primitives_closed_form_and_fd(oracle_mod):
+    rng = np.random.default_rng(17)
+    th = rng.normal(0, 1, (4, 9)) + 2 * np.eye(3).reshape(-1)
+    loss, grad = run(oracle_mod, MATPROG, th)
+    loss_d, grad_d = run(oracle_mod, MATPROG, th, mode=2)
+    for b in range(4):
+        A = th[b].reshape(3, 3)
+        S = A @ A.T + np.eye(3)
+        B2 = A[0:2, 1:3]
+        v = 0.5 * ((A @ np.array([1.0, -2.0, 0.5])) @ np.array([0.3, 0.2, 0.1]))
+        ref = (np.linalg.det(A) + np.log(np.linalg.det(S)) + np.trace(np.linalg.inv(S) @ A)
+               + np.linalg.inv(B2)[0, 1] + v + np.trace(A[0, 0] * A))
+        assert_rel(loss[b], ref, 1e-12)
+        fd = central_fd(oracle_mod, MATPROG, th[b], ())
+        assert_rel(grad[b], fd, 1e-7, scale=np.max(np.abs(grad[b])))
+        assert_rel(grad[b], grad_d[b], 1e-13, scale=np.max(np.abs(grad[b])))
+    # det: d det A / dA = det(A) A^-T (Appendix C); pin on a non-symmetric matrix
+    DET = "(model (params a b c d e f g h i) (det (matrix 3 3 a b c d e f g h i)))"
+    A = np.array([[2.0, -1.0, 0.5], [0.3, 1.7, -0.2], [1.1, 0.4, 3.0]])
+    _, gd = run(oracle_mod, DET, A.reshape(1, 9))
+    np.testing.assert_allclose(gd[0].reshape(3, 3), np.linalg.det(A) * np.linalg.inv(A).T, rtol=1e-13, atol=1e-13)
+    # inv of a 5x5 (Gauss-Jordan path): d/dA sum(W * inv(A)) = -A^-T W A^-T
+    n = 5
+    A5 = np.eye(n) * 3 + rng.normal(0, 0.5, (n, n))
+    Wm = rng.normal(0, 1, (n, n))
+    names = " ".join(f"p{k}" for k in range(n * n))
+    wel = " ".join(repr(float(x)) for x in Wm.reshape(-1))
+    INV5 = (f"(model (params {names}) (trace (matmul (matrix {n} {n} {wel}) "
+            f"(transpose (inv (matrix {n} {n} {names}))))))")
+    l5, g5 = run(oracle_mod, INV5, A5.reshape(1, -1))
+    Ai = np.linalg.inv(A5)
+    assert_rel(l5[0], np.sum(Wm * Ai), 1e-12)
+    np.testing.assert_allclose(g5[0].reshape(n, n), -Ai.T @ Wm @ Ai.T, rtol=1e-11, atol=1e-12)
+
+
+# --------------------------------------------- primitive rules and edge cases
+def test_clamps_abs_and_pow_int(oracle_mod):
+    # log/sqrt: forward on max(x, 1e-8), zero gradient unless x > 1e-8 (Appendix C)
+    LOGP = "(model (params x) (log x))"
+    SQRTP = "(model (params x) (sqrt x))"
+    xs = np.array([[1e-8], [5e-9], [-1.0], [2e-8], [3.0]])
+    l, g = run(oracle_mod, LOGP, xs)
+    np.testing.assert_array_equal(l[:3], np.log(1e-8))
+    np.testing.assert_array_equal(g[:3, 0], 0.0)
+    np.testing.assert_allclose(g[3:, 0], 1 / xs[3:, 0], rtol=1e-15)
+    l, g = run(oracle_mod, SQRTP, xs)
+    np.testing.assert_array_equal(l[:3], math.sqrt(1e-8))
+    np.testing.assert_array_equal(g[:3, 0], 0.0)
+    np.testing.assert_allclose(g[3:, 0], 0.5 / np.sqrt(xs[3:, 0]), rtol=1e-15)
+    # abs'(0) = 0
+    l, g = run(oracle_mod, "(model (params x) (abs x))", [[0.0], [-2.0], [3.0]])
+    np.testing.assert_array_equal(g[:, 0], [0.0, -1.0, 1.0])
+    # integer power by repeated multiplication; derivative n a^(n-1), finite at 0
+    l, g = run(oracle_mod, "(model (params x) (pow x 3))", [[0.0], [-1.5], [2.0]])
+    np.testing.assert_array_equal(l, [0.0, -3.375, 8.0])
+    np.testing.assert_array_equal(g[:, 0], [0.0, 6.75, 12.0])
+    l, g = run(oracle_mod, "(model (params x) (pow x 0))", [[0.0], [5.0]])
+    np.testing.assert_array_equal(l, [1.0, 1.0])
+    np.testing.assert_array_equal(g[:, 0], [0.0, 0.0])
+    # general pow (Appendix C): a^e, d/da = e z / a, d/de = z ln a
+    l, g = run(oracle_mod, "(model (params a e) (pow a e))", [[2.0, 1.5]])
+    z = 2.0 ** 1.5
+    np.testing.assert_allclose(g[0], [1.5 * z / 2.0, z * math.log(2.0)], rtol=1e-15)
+
+
+def test_nary_forms(oracle_mod):
+    # Appendix C: sub z = x0 - sum(x_i), div z = x0 / prod(x_i); single-argument - and / negate / invert
+    P = "(model (params a b c) (+ (- a b c) (/ a b c) (- a) (/ b) (* a b c)))"
+    th = np.array([[1.5, -2.0, 0.7]])
+    l, g = run(oracle_mod, P, th)
+    a, b, c = th[0]
+    assert_rel(l[0], (a - b - c) + a / (b * c) - a + 1 / b + a * b * c, 1e-15)
+    ga = 1 + 1 / (b * c) - 1 + b * c
+    gb = -1 - a / (b * b * c) - 1 / (b * b) + a * c
+    gc = -1 - a / (b * c * c) + a * b
+    assert_rel(g[0], [ga, gb, gc], 1e-14, scale=max(abs(ga), abs(gb), abs(gc)))
+
+
+def test_per_lane_branch_gating(oracle_mod):
+    # Property 1: a parameter that appears only in a test gets no gradient; the taken side gets it
+    P = "(model (params a t) (if (< t 0.0) (* a a) (* 3.0 a)))"
+    l, g = run(oracle_mod, P, [[2.0, -1.0], [2.0, 1.0]])
+    np.testing.assert_array_equal(l, [4.0, 6.0])
+    np.testing.assert_array_equal(g, [[4.0, 0.0], [3.0, 0.0]])
+    # an untaken side that would be infinite never leaks into the gradient
+    P2 = "(model (params a) (if (> a 0.0) (log a) (* 2.0 a)))"
+    l, g = run(oracle_mod, P2, [[0.5], [-1.0]])
+    np.testing.assert_allclose(g[:, 0], [2.0, 2.0])
+
+
+def test_invariants(oracle_mod):
+    # a parameter-free program has zero gradient
+    l, g = run(oracle_mod, "(model (params a b) (+ (exp 1.0) (obs 0)))", [[1.0, 2.0], [3.0, 4.0]], [5.0])
+    np.testing.assert_array_equal(g, 0.0)
+    np.testing.assert_allclose(l, math.e + 5.0)
+    # identical lanes give identical outputs; lane order does not matter
+    w = W.random_exprs(n_programs=3, B=6, n_points=32, seed=5)[2]
+    p = np.repeat(w.params[:1], 4, axis=0)
+    l, g = run(oracle_mod, w.program, p, w.obs)
+    assert np.all(l == l[0]) and np.all(g == g[0])
+    perm = np.array([3, 0, 5, 1, 4, 2])
+    l1, g1 = run(oracle_mod, w.program, w.params, w.obs)
+    l2, g2 = run(oracle_mod, w.program, w.params[perm], w.obs)
+    np.testing.assert_array_equal(l1[perm], l2)
+    np.testing.assert_array_equal(g1[perm], g2)
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3, 4, 5])
+def test_reverse_mode_equals_dual_numbers(oracle_mod, cfg):
+    if cfg == 2:
+        ws = W.random_exprs(n_programs=10, B=3, n_points=64, seed=2)
+    elif cfg == 5:
+        ws = [W.kalman_rand8(B=2, T=40)]
+    elif cfg == 4:
+        ws = [W.kalman_cv4(B=3, T=60)]
+    else:
+        ws = [W.config(cfg, B=4)]
+    for w in ws:
+        l1, g1 = run(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend, mode=1)
+        l2, g2 = run(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend, mode=2)
+        np.testing.assert_array_equal(l1, l2)
+        s = np.max(np.abs(g1), axis=1, keepdims=True)
+        assert np.max(np.abs(g1 - g2) / s) < 1e-13
+
+
+def test_magnitude_mode(oracle_mod):
+    # the magnitude mode propagates absolute values: for 3a - 2a the gradient is 1 and
+    # the terms it sums have size 3 + 2
+    l, g, m = oracle_mod.run("(model (params a) (- (* 3.0 a) (* 2.0 a)))", np.array([[1.7]]), np.zeros(0),
+                             magnitudes=True)
+    np.testing.assert_array_equal(g, [[1.0]])
+    np.testing.assert_array_equal(m, [[5.0]])
+    # a product rule: d/da (a * (-b)) = -b, d/db = -a; magnitudes |b|, |a|
+    l, g, m = oracle_mod.run("(model (params a b) (* a (- b)))", np.array([[2.0, -3.0]]), np.zeros(0),
+                             magnitudes=True)
+    np.testing.assert_array_equal(g, [[3.0, -2.0]])
+    np.testing.assert_array_equal(m, [[3.0, 2.0]])
+    # magnitudes bound the gradient on every workload
+    w = W.kalman_cv4(B=3, T=30)
+    l, g, m = oracle_mod.run(w.program, w.params, w.obs, magnitudes=True)
+    assert np.all(m >= np.abs(g) * (1 - 1e-12))
+
+
+def test_threads_do_not_change_results(oracle_mod):
+    w = W.kalman_cv4(B=13, T=30)
+    a = oracle_mod.run(w.program, w.params, w.obs, nthreads=1)
+    b = oracle_mod.run(w.program, w.params, w.obs, nthreads=5)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
+
+
+# ------------------------------------------------------ bytecode (section 7)
+def test_bytecode_workloads(oracle_mod):
+    # W1 scalar expression: exp(a) * sin(b) - log(c) / 2
+    W1 = "PARAM 0\nEXP\nPARAM 1\nSIN\nMUL\nPARAM 2\nLOG\nPUSH 2.0\nDIV\nSUB\n"
+    th = np.array([[0.3, 1.1, 2.5]])
+    l, g = run(oracle_mod, W1, th, frontend=1)
+    a, b, c = th[0]
+    assert_rel(l[0], math.exp(a) * math.sin(b) - math.log(c) / 2, 1e-15)
+    assert_rel(g[0], [math.exp(a) * math.sin(b), math.exp(a) * math.cos(b), -0.5 / c], 1e-15)
+    # W2 counted loop: x <- x * a + b, 7 times from x = 1
+    W2 = "PUSH 1.0\nSTORE 0\nLOOP 7\nLOAD 0\nPARAM 0\nMUL\nPARAM 1\nADD\nSTORE 0\nEND\nLOAD 0\n"
+    th = np.array([[0.9, 0.2]])
+    l, g = run(oracle_mod, W2, th, frontend=1)
+    x, dxa, dxb = 1.0, 0.0, 0.0
+    for _ in range(7):
+        dxa, dxb = dxa * 0.9 + x, dxb * 0.9 + 1.0
+        x = x * 0.9 + 0.2
+    assert_rel(l[0], x, 1e-15)
+    assert_rel(g[0], [dxa, dxb], 1e-14)
+    # W3 branch (lane mask): a < b ? a*b : a+b
+    W3 = "PARAM 0\nPARAM 1\nLT\nPARAM 0\nPARAM 1\nMUL\nPARAM 0\nPARAM 1\nADD\nSEL\n"
+    l, g = run(oracle_mod, W3, [[1.0, 3.0], [4.0, 2.0]], frontend=1)
+    np.testing.assert_array_equal(l, [3.0, 6.0])
+    np.testing.assert_array_equal(g, [[3.0, 1.0], [1.0, 1.0]])
+    # W4 dot product and LOOP 0
+    W4 = "PARAM 0\nPARAM 1\nPUSH 2.0\nPUSH 3.0\nDOT 2\nLOOP 0\nPUSH 9.0\nEND\n"
+    l, g = run(oracle_mod, W4, [[0.5, -1.0]], frontend=1)
+    np.testing.assert_array_equal(l, [0.5 * 2 - 3.0])
+    np.testing.assert_array_equal(g, [[2.0, 3.0]])
+
+
+def test_errors_are_reported(oracle_mod):
+    with pytest.raises(oracle_mod.OracleError):
+        run(oracle_mod, "(model (params a) (+ a", [[1.0]])
+    with pytest.raises(oracle_mod.OracleError):
+        run(oracle_mod, "(model (params a) (matmul (identity 2) (identity 3)))", [[1.0]])
+    with pytest.raises(oracle_mod.OracleError):
+        run(oracle_mod, "PARAM 0\nADD\n", [[1.0]], frontend=1)

@@ -1,0 +1,426 @@
+"""Seeded synthetic workloads for the NDVM tape-replay path.
+
+This module only *synthesises inputs*: program texts, observation vectors and
+per-lane parameter draws, from numpy's PCG64 generator with fixed seeds.  It holds
+none of the method's arithmetic (no tape, no adjoint, no loss reduction), and it is
+the only code shared by the product's tests/benchmark and the oracle.  Simulating
+the data-generating process (an Euler trajectory, a linear-Gaussian state-space
+model, a random expression evaluated at its hidden constants) is part of the input
+recipe, done here with plain numpy.
+
+Five workloads, shaped like the paper's (sections 6-7 and Appendix A):
+
+  1 exp-decay      y = a exp(-b t) + c, 50 points, MSE, P=3, B=64
+  2 random exprs   200 programs (+ - * / exp log|x| sin pow-int, depth <= 6,
+                   1-8 constants), 256 points, MSE, B=4096 lanes per program
+  3 logistic       bytecode, explicit Euler dx/dt = r x (1 - x/K), 1000 steps,
+                   dt = 0.01, 100 observations, MSE, P=2, B=16384
+  4 kalman-4       4-state constant-velocity Kalman NLL, 2-d obs, T=200, P=4, B=8192
+  5 kalman-8       8-state random stable Kalman NLL, 3-d obs, T=1000, P=12, B=65536
+
+Every generator takes the sizes as arguments, so tests can build small instances
+of the same recipe.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+FRONTEND_SCHEME = 0
+FRONTEND_BYTECODE = 1
+
+
+@dataclass
+class Workload:
+    name: str
+    program: str            # program text (the single source of truth for both paths)
+    frontend: int           # 0 Scheme-style, 1 stack bytecode
+    params: np.ndarray      # (B, P) float64 lane parameters
+    obs: np.ndarray         # (n_obs,) float64 observations shared by all lanes
+    truth: np.ndarray       # (P,) hidden parameters used to synthesise obs
+    meta: dict = field(default_factory=dict)
+
+    @property
+    def B(self) -> int:
+        return int(self.params.shape[0])
+
+    @property
+    def P(self) -> int:
+        return int(self.params.shape[1])
+
+
+def _fmt(x: float) -> str:
+    """Shortest round-tripping decimal for a double, always with a '.' or exponent."""
+    s = repr(float(x))
+    if "e" not in s and "." not in s and "inf" not in s and "nan" not in s:
+        s += ".0"
+    return s
+
+
+# --------------------------------------------------------------------------
+# 1. exponential decay
+# --------------------------------------------------------------------------
+def exp_decay(B: int = 64, n_points: int = 50, seed: int = 1234) -> Workload:
+    rng = np.random.default_rng(seed)
+    truth = np.array([1.3, 0.8, 0.9])
+    t = rng.uniform(0.0, 5.0, n_points)
+    y = truth[0] * np.exp(-truth[1] * t) + truth[2] + rng.normal(0.0, 0.05, n_points)
+    obs = np.empty(2 * n_points)
+    obs[0::2] = t
+    obs[1::2] = y
+    params = rng.normal(1.0, 0.3, (B, 3))
+    program = (
+        ";; exponential decay y = a exp(-b t) + c, mean squared error over the data axis\n"
+        "(model (params a b c)\n"
+        f"  (/ (data-sum {n_points} 2\n"
+        "       (let ((r (- (+ (* a (exp (- (* b (dobs 0))))) c) (dobs 1))))\n"
+        "         (* r r)))\n"
+        f"     {_fmt(float(n_points))}))\n"
+    )
+    return Workload("exp_decay", program, FRONTEND_SCHEME, params, obs, truth,
+                    {"n_points": n_points})
+
+
+# --------------------------------------------------------------------------
+# 2. random expression programs (the paper's typed program generator, section 6)
+# --------------------------------------------------------------------------
+# Grammar: + - * / exp log|x| sin pow-int over x and constants theta_k.
+# Domain guards follow the paper's generator: a division denominator d is wrapped
+# to 1 + d*d, a log argument a to 1 + a*a (inside log|.|), an exp argument a is
+# squashed to a / (1 + a*a).  A program is kept only if every intermediate value
+# stays within 1e4 in magnitude at the hidden constants and at sampled lanes.
+
+_BIN = ("+", "-", "*", "/")
+_UN = ("exp", "log", "sin", "pow")
+
+
+class _Gen:
+    def __init__(self, rng, max_depth, max_consts):
+        self.rng = rng
+        self.max_depth = max_depth
+        self.max_consts = max_consts
+        self.nconst = 0
+
+    def leaf(self):
+        # x or a constant
+        if self.rng.random() < 0.5 or self.nconst == 0:
+            if self.nconst < self.max_consts and self.rng.random() < 0.6:
+                k = self.nconst
+                self.nconst += 1
+                return ("c", k)
+            if self.nconst > 0 and self.rng.random() < 0.3:
+                return ("c", int(self.rng.integers(0, self.nconst)))
+        return ("x",)
+
+    def expr(self, depth):
+        p_leaf = 0.15 + 0.85 * (depth / self.max_depth) ** 2
+        if depth >= self.max_depth or (depth > 0 and self.rng.random() < p_leaf):
+            return self.leaf()
+        if self.rng.random() < 0.65:
+            op = _BIN[int(self.rng.integers(0, 4))]
+            return (op, self.expr(depth + 1), self.expr(depth + 1))
+        op = _UN[int(self.rng.integers(0, 4))]
+        if op == "pow":
+            return ("pow", self.expr(depth + 1), int(self.rng.integers(2, 4)))
+        return (op, self.expr(depth + 1))
+
+
+def _expr_text(e, names=None) -> str:
+    """Program text of a generator tree; guarded operands are let-bound once."""
+    if names is None:
+        names = [0]
+
+    def fresh():
+        names[0] += 1
+        return f"g{names[0]}"
+
+    k = e[0]
+    if k == "x":
+        return "x"
+    if k == "c":
+        return f"t{e[1]}"
+    if k in ("+", "-", "*"):
+        return f"({k} {_expr_text(e[1], names)} {_expr_text(e[2], names)})"
+    if k == "/":
+        a = _expr_text(e[1], names)
+        d = _expr_text(e[2], names)
+        v = fresh()
+        return f"(let (({v} {d})) (/ {a} (+ 1.0 (* {v} {v}))))"
+    if k == "exp":
+        a = _expr_text(e[1], names)
+        v = fresh()
+        return f"(let (({v} {a})) (exp (/ {v} (+ 1.0 (* {v} {v})))))"
+    if k == "log":
+        a = _expr_text(e[1], names)
+        v = fresh()
+        return f"(let (({v} {a})) (log (abs (+ 1.0 (* {v} {v})))))"
+    if k == "sin":
+        return f"(sin {_expr_text(e[1], names)})"
+    if k == "pow":
+        return f"(pow {_expr_text(e[1], names)} {e[2]})"
+    raise ValueError(k)
+
+
+def _expr_eval(e, x, th, guard):
+    """numpy evaluation of the generator's own tree (data synthesis only)."""
+    k = e[0]
+    if k == "x":
+        v = x
+    elif k == "c":
+        v = th[..., e[1]][..., None] * np.ones_like(x)
+    elif k in _BIN:
+        a = _expr_eval(e[1], x, th, guard)
+        b = _expr_eval(e[2], x, th, guard)
+        if k == "+":
+            v = a + b
+        elif k == "-":
+            v = a - b
+        elif k == "*":
+            v = a * b
+        else:
+            v = a / (1.0 + b * b)
+    elif k == "exp":
+        a = _expr_eval(e[1], x, th, guard)
+        v = np.exp(a / (1.0 + a * a))
+    elif k == "log":
+        a = _expr_eval(e[1], x, th, guard)
+        v = np.log(np.abs(1.0 + a * a))
+    elif k == "sin":
+        v = np.sin(_expr_eval(e[1], x, th, guard))
+    elif k == "pow":
+        v = _expr_eval(e[1], x, th, guard) ** e[2]
+    else:
+        raise ValueError(k)
+    guard.append(float(np.max(np.abs(v))) if v.size else 0.0)
+    return v
+
+
+def _uses_x(e) -> bool:
+    if e[0] == "x":
+        return True
+    if e[0] == "c":
+        return False
+    return any(_uses_x(s) for s in e[1:] if isinstance(s, tuple))
+
+
+def _size(e) -> int:
+    if e[0] in ("x", "c"):
+        return 1
+    return 1 + sum(_size(s) for s in e[1:] if isinstance(s, tuple))
+
+
+def random_program(rng, n_points: int, max_depth: int = 6, max_consts: int = 8,
+                   guard_lanes: int = 32):
+    """Draw one accepted random-expression program; returns (text, tree, theta*, x, y)."""
+    while True:
+        g = _Gen(rng, max_depth, max_consts)
+        tree = g.expr(0)
+        if g.nconst < 1 or not _uses_x(tree) or _size(tree) < 4:
+            continue
+        P = g.nconst
+        theta = rng.uniform(-2.0, 2.0, P)
+        x = rng.uniform(-2.0, 2.0, n_points)
+        lanes = theta + rng.normal(0.0, 0.3, (guard_lanes, P))
+        with np.errstate(all="ignore"):
+            guard = []
+            f_star = _expr_eval(tree, x[None, :], theta[None, :], guard)[0]
+            _expr_eval(tree, x[None, :], lanes, guard)
+        if not all(np.isfinite(guard)) or max(guard) > 1e4:
+            continue
+        y = f_star + rng.normal(0.0, 0.05, n_points)
+        names = " ".join(f"t{k}" for k in range(P))
+        body = _expr_text(tree)
+        text = (
+            ";; random expression program, mean squared error over the data axis\n"
+            f"(model (params {names})\n"
+            f"  (/ (data-sum {n_points} 2\n"
+            f"       (let* ((x (dobs 0)) (r (- {body} (dobs 1))))\n"
+            "         (* r r)))\n"
+            f"     {_fmt(float(n_points))}))\n"
+        )
+        return text, tree, theta, x, y
+
+
+def random_exprs(n_programs: int = 200, B: int = 4096, n_points: int = 256, seed: int = 1234,
+                 max_depth: int = 6):
+    """List of Workloads (one per program)."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n_programs):
+        text, tree, theta, x, y = random_program(rng, n_points, max_depth=max_depth)
+        obs = np.empty(2 * n_points)
+        obs[0::2] = x
+        obs[1::2] = y
+        params = theta + rng.normal(0.0, 0.3, (B, theta.size))
+        out.append(Workload(f"random_expr_{i}", text, FRONTEND_SCHEME, params, obs, theta,
+                            {"n_points": n_points, "tree_size": _size(tree)}))
+    return out
+
+
+# --------------------------------------------------------------------------
+# 3. logistic growth, stack bytecode (section 7's second client)
+# --------------------------------------------------------------------------
+def logistic_bytecode(n_obs: int = 100, every: int = 10, dt: float = 0.01, x0: float = 0.1) -> str:
+    lines = [
+        "; logistic growth dx/dt = r x (1 - x/K), explicit Euler; MSE against observations",
+        "PARAM 0", "STORE 0            ; r",
+        "PARAM 1", "STORE 1            ; K",
+        f"PUSH {_fmt(x0)}", "STORE 2            ; x",
+        "PUSH 0.0", "STORE 3            ; squared-error accumulator",
+        f"LOOP {n_obs}",
+        f"  LOOP {every}",
+        "    LOAD 2", "    LOAD 0", "    LOAD 2", "    MUL            ; r x",
+        "    PUSH 1.0", "    LOAD 2", "    LOAD 1", "    DIV            ; x / K",
+        "    SUB            ; 1 - x/K", "    MUL            ; r x (1 - x/K)",
+        f"    PUSH {_fmt(dt)}", "    MUL", "    ADD            ; x + dt f(x)", "    STORE 2",
+        "  END",
+        "  LOAD 3", "  LOAD 2", "  OBSN", "  SUB", "  DUP", "  MUL", "  ADD", "  STORE 3",
+        "END",
+        "LOAD 3", f"PUSH {_fmt(float(n_obs))}", "DIV",
+    ]
+    return "\n".join(lines) + "\n"
+
+
+def logistic(B: int = 16384, n_obs: int = 100, every: int = 10, seed: int = 1234) -> Workload:
+    rng = np.random.default_rng(seed)
+    truth = np.array([0.8, 1.0])
+    dt, x = 0.01, 0.1
+    ys = []
+    for _ in range(n_obs):
+        for _ in range(every):
+            x = x + dt * (truth[0] * x * (1.0 - x / truth[1]))
+        ys.append(x)
+    obs = np.array(ys) + rng.normal(0.0, 0.01, n_obs)
+    params = truth * np.exp(0.25 * rng.normal(0.0, 1.0, (B, 2)))
+    return Workload("logistic", logistic_bytecode(n_obs, every, dt), FRONTEND_BYTECODE, params, obs,
+                    truth, {"steps": n_obs * every, "n_obs": n_obs})
+
+
+# --------------------------------------------------------------------------
+# 4/5. Kalman filter negative log-likelihood (prediction-error decomposition)
+# --------------------------------------------------------------------------
+def _matrix_text(M) -> str:
+    r, c = M.shape
+    el = " ".join(_fmt(v) for v in M.reshape(-1))
+    return f"(matrix {r} {c} {el})"
+
+
+_KALMAN_LOOP = """(define (kalman-nll Q R P0 T)
+  (let loop ((t 0) (x (zeros {n} 1)) (P P0) (nll 0.0))
+    (if (= t T)
+        nll
+        (let* ((xp (matmul F x))
+               (Pp (m+ (matmul (matmul F P) (transpose F)) Q))
+               (v (m- (obs-vec (* {m} t) {m}) (matmul H xp)))
+               (PHt (matmul Pp (transpose H)))
+               (S (m+ (matmul H PHt) R))
+               (Si (inv S))
+               (K (matmul PHt Si))
+               (xn (m+ xp (matmul K v)))
+               (Pn (m- Pp (matmul K (matmul H Pp))))
+               (term (* 0.5 (+ (logdet S) (mref (matmul (transpose v) (matmul Si v)) 0 0) {c}))))
+          (loop (+ t 1) xn Pn (+ nll term))))))
+"""
+
+
+def _simulate_lgssm(rng, F, H, Q, R, P0, T):
+    n = F.shape[0]
+    x = rng.multivariate_normal(np.zeros(n), P0)
+    ys = []
+    for _ in range(T):
+        x = F @ x + rng.multivariate_normal(np.zeros(n), Q)
+        ys.append(H @ x + rng.multivariate_normal(np.zeros(H.shape[0]), R))
+    return np.concatenate(ys)
+
+
+def kalman_cv4(B: int = 8192, T: int = 200, seed: int = 1234) -> Workload:
+    """4-state constant-velocity model (px, py, vx, vy), dt = 1, 2-d position observations."""
+    rng = np.random.default_rng(seed)
+    F = np.array([[1, 0, 1, 0], [0, 1, 0, 1], [0, 0, 1, 0], [0, 0, 0, 1]], dtype=float)
+    H = np.array([[1, 0, 0, 0], [0, 1, 0, 0]], dtype=float)
+    truth = np.log(np.array([0.5, 0.4, 1.0, 0.8]))
+    qx, qy, rx, ry = np.exp(2 * truth)
+    Q = np.array([[qx / 3, 0, qx / 2, 0], [0, qy / 3, 0, qy / 2], [qx / 2, 0, qx, 0], [0, qy / 2, 0, qy]])
+    R = np.diag([rx, ry])
+    P0 = 10.0 * np.eye(4)
+    obs = _simulate_lgssm(rng, F, H, Q, R, P0, T)
+    params = truth + rng.normal(0.0, 0.5, (B, 4))
+    m = 2
+    program = (
+        ";; 4-state constant-velocity Kalman filter, Gaussian negative log-likelihood\n"
+        f"(define F {_matrix_text(F)})\n"
+        f"(define H {_matrix_text(H)})\n"
+        + _KALMAN_LOOP.format(n=4, m=m, c=_fmt(m * math.log(2 * math.pi)))
+        + "(model (params lqx lqy lrx lry)\n"
+        "  (let* ((qx (exp (* 2.0 lqx))) (qy (exp (* 2.0 lqy)))\n"
+        "         (rx (exp (* 2.0 lrx))) (ry (exp (* 2.0 lry)))\n"
+        "         (Q (matrix 4 4 (/ qx 3.0) 0 (/ qx 2.0) 0\n"
+        "                        0 (/ qy 3.0) 0 (/ qy 2.0)\n"
+        "                        (/ qx 2.0) 0 qx 0\n"
+        "                        0 (/ qy 2.0) 0 qy))\n"
+        "         (R (matrix 2 2 rx 0 0 ry)))\n"
+        f"    (kalman-nll Q R (mscale 10.0 (identity 4)) {T})))\n"
+    )
+    return Workload("kalman_cv4", program, FRONTEND_SCHEME, params, obs, truth, {"T": T, "n": 4, "m": m})
+
+
+def random_stable_matrix(rng, n: int, radius: float = 0.95) -> np.ndarray:
+    A = rng.normal(0.0, 1.0, (n, n))
+    rho = float(np.max(np.abs(np.linalg.eigvals(A))))
+    return A * (radius / rho)
+
+
+def kalman_rand8(B: int = 65536, T: int = 1000, seed: int = 1234, n: int = 8, m: int = 3) -> Workload:
+    """n-state linear-Gaussian model, random transition with spectral radius 0.95, H = [I_m 0]."""
+    rng = np.random.default_rng(seed)
+    F = random_stable_matrix(rng, n)
+    H = np.zeros((m, n))
+    H[:, :m] = np.eye(m)
+    truth = np.concatenate([np.log(rng.uniform(0.1, 0.3, n)), np.log(np.full(m, 0.5)), [0.0]])
+    Q = np.diag(np.exp(2 * truth[:n]))
+    R = np.diag(np.exp(2 * truth[n:n + m]))
+    P0 = np.exp(2 * truth[-1]) * np.eye(n)
+    obs = _simulate_lgssm(rng, F, H, Q, R, P0, T)
+    params = truth + rng.normal(0.0, 0.5, (B, n + m + 1))
+    qn = " ".join(f"lq{i}" for i in range(n))
+    rn = " ".join(f"lr{i}" for i in range(m))
+    qdiag = []
+    for i in range(n):
+        row = ["0"] * n
+        row[i] = f"(exp (* 2.0 lq{i}))"
+        qdiag.append(" ".join(row))
+    rdiag = []
+    for i in range(m):
+        row = ["0"] * m
+        row[i] = f"(exp (* 2.0 lr{i}))"
+        rdiag.append(" ".join(row))
+    program = (
+        f";; {n}-state random stable Kalman filter, {m}-d observations, Gaussian negative log-likelihood\n"
+        f"(define F {_matrix_text(F)})\n"
+        f"(define H {_matrix_text(H)})\n"
+        + _KALMAN_LOOP.format(n=n, m=m, c=_fmt(m * math.log(2 * math.pi)))
+        + f"(model (params {qn} {rn} lp0)\n"
+        f"  (kalman-nll (matrix {n} {n} " + "\n      ".join(qdiag) + ")\n"
+        f"              (matrix {m} {m} " + " ".join(rdiag) + ")\n"
+        f"              (mscale (exp (* 2.0 lp0)) (identity {n}))\n"
+        f"              {T}))\n"
+    )
+    return Workload(f"kalman_rand{n}", program, FRONTEND_SCHEME, params, obs, truth,
+                    {"T": T, "n": n, "m": m, "F": F})
+
+
+def config(i: int, **kw):
+    """Workload(s) of the five configurations at their full sizes (or overridden sizes)."""
+    if i == 1:
+        return exp_decay(**kw)
+    if i == 2:
+        return random_exprs(**kw)
+    if i == 3:
+        return logistic(**kw)
+    if i == 4:
+        return kalman_cv4(**kw)
+    if i == 5:
+        return kalman_rand8(**kw)
+    raise ValueError(i)
