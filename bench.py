@@ -1,0 +1,277 @@
+"""Benchmark: lane value+grad evaluations per second of the NDVM tape replay on GB300.
+
+One step = the whole hot path over one batch: 200 seeded random-expression programs
+(grammar + - * / exp log|x| sin pow-int, depth <= 6, 1-8 constants), each replayed
+forward and in reverse over B = 4096 parameter lanes and 256 data points (MSE loss)
+-- 819,200 lane value+grad evaluations.  Inputs are resident in HBM before the timed
+region; L2 is flushed between timed steps.  Prints one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+--impl reference times the oracle (the plain CPU reference evaluator) on the host
+cores instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+N_PROGRAMS, B_LANES, N_POINTS, SEED = 200, 4096, 256, 1234
+METRIC = "lane value+grad evals/sec (fp64, 1 GB300) and % of FP64/HBM roofline"
+UNIT = "lane-evals/s"
+WORKLOAD = (f"random-expression programs: {N_PROGRAMS} programs x {B_LANES} lanes x {N_POINTS} points, "
+            "MSE, fp64 value+grad")
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples taken during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int):
+    """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program."""
+    import oracle
+    oracle.build()
+    t0 = time.perf_counter()
+    n = 0
+    for w in progs:
+        oracle.run(w.program, w.params[:lanes_per_prog], w.obs, frontend=w.frontend, nthreads=nthreads)
+        n += lanes_per_prog
+    return n, time.perf_counter() - t0
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    cores = os.cpu_count() or 1
+    progs = W.random_exprs(n_programs=N_PROGRAMS, B=B_LANES, n_points=N_POINTS, seed=SEED)
+    lanes = args.ref_lanes
+    for _ in range(args.warmup):
+        oracle_sample_time(progs[:4], 2, cores)
+    times, n = [], 0
+    for _ in range(args.steps):
+        n, dt = oracle_sample_time(progs, lanes, cores)
+        times.append(dt)
+    ms = 1e3 * float(np.mean(times))
+    value = n / (ms * 1e-3)
+    sample = f"{lanes} lanes of each of the {N_PROGRAMS} programs ({n} lane evals per step), all points"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic", "config": {"workload": WORKLOAD, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
+    ap.add_argument("--ref-lanes", type=int, default=48, help="oracle lanes per program per reference step")
+    ap.add_argument("--cpu-lanes", type=int, default=48, help="oracle lanes per program for cpu_baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import paper_2607_03574_gb300 as nd
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    nd.load()
+
+    # ---- workload: programs traced once on the host; inputs resident in HBM
+    progs = W.random_exprs(n_programs=N_PROGRAMS, B=B_LANES, n_points=N_POINTS, seed=SEED + rank)
+    t0 = time.perf_counter()
+    tapes = [nd.trace_build(w.program, w.frontend) for w in progs]
+    trace_s = time.perf_counter() - t0
+    params = [torch.tensor(w.params, dtype=torch.float64, device=dev) for w in progs]
+    obs = [torch.tensor(w.obs, dtype=torch.float64, device=dev) for w in progs]
+    loss = [torch.empty(w.B, dtype=torch.float64, device=dev) for w in progs]
+    grad = [torch.empty_like(p) for p in params]
+    flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
+    stream = torch.cuda.current_stream(dev)
+    work = 0.0
+    for tp, w in zip(tapes, progs):
+        c = tp.cost()
+        work += (c["work_fwd"] + c["work_rev"]) * w.B
+
+    def step():
+        for k in range(N_PROGRAMS):
+            nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    peak_flops = nd.measure_fp64_peak()
+
+    clocks = ClockSampler(local)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    l0 = nd.launch_count()
+    step_ms = []
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    launches = nd.launch_count() - l0
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = float(np.mean(step_ms))
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    clk = clocks.stop()
+    lanes_per_step = N_PROGRAMS * B_LANES * world
+    value = lanes_per_step / (ms * 1e-3)
+
+    # ---- end to end through the host-buffer entry point (pinned host memory)
+    hp = [torch.tensor(w.params, dtype=torch.float64).pin_memory().numpy() for w in progs]
+    ho = [torch.tensor(w.obs, dtype=torch.float64).pin_memory().numpy() for w in progs]
+    h2d = sum(a.nbytes for a in hp) + sum(a.nbytes for a in ho)
+    d2h = sum(w.B * 8 * (1 + w.P) for w in progs)
+
+    def e2e_step():
+        for k in range(N_PROGRAMS):
+            nd.value_and_grad_host(tapes[k], hp[k], ho[k])
+
+    e2e_step()
+    e2e_times = []
+    for _ in range(max(2, args.steps // 2)):
+        t1 = time.perf_counter()
+        e2e_step()
+        e2e_times.append(time.perf_counter() - t1)
+    e2e_value = lanes_per_step / float(np.mean(e2e_times)) if world == 1 else None
+
+    # ---- roofline of the replay kernel: algorithmic FP64 work / kernel time
+    achieved = 2.0 * work / (ms * 1e-3)  # flop/s (2 per DFMA-equivalent), kernels only
+    roofline = {
+        "bound": "alu", "achieved": achieved / 1e12, "peak": peak_flops / 1e12, "unit": "TFLOP/s",
+        "frac": achieved / peak_flops, "traffic": None,
+        "peak_source": "FP64 FMA rate measured in this process (8 chains/thread, 4x256 threads/SM)",
+        "work_dfma_per_step": work,
+    }
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        oracle_sample_time(progs[:2], 2, cores)
+        n, dt = oracle_sample_time(progs, args.cpu_lanes, cores)
+        cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"{args.cpu_lanes} lanes of each of the {N_PROGRAMS} programs ({n} lane evals, {dt:.1f} s)"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "programs": N_PROGRAMS, "lanes_per_program": B_LANES,
+                       "points": N_POINTS, "seed": SEED, "l2": "flushed (256 MB write) before every timed step",
+                       "parallelism": f"lanes sharded, dp{world}"},
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches // max(1, args.steps) * args.steps,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "clocks": clk,
+            "wall_s_timed": wall,
+            "trace_build_s": trace_s,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

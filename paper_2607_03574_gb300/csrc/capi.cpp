@@ -1,0 +1,371 @@
+// C ABI implementation: tape objects, device caches, launch configuration.
+#include <cuda_runtime.h>
+
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "plan.h"
+#include "replay.h"
+#include "status.h"
+#include "tape.h"
+
+using namespace ndvm;
+
+namespace {
+
+thread_local std::string g_last_error;
+std::mutex g_launch_mu;
+unsigned long long g_launches = 0;
+
+ndvm_status fail(ndvm_status s, const std::string& m) {
+  g_last_error = m;
+  return s;
+}
+ndvm_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(NDVM_E_CUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+struct DevPlan {
+  DInst* code = nullptr;
+  int32_t* args = nullptr;
+  double* consts_d = nullptr;
+  float* consts_f = nullptr;
+};
+
+struct DevCache {
+  DevPlan grad, value;
+  int* err = nullptr;
+  // buffers for the host-pointer entry point
+  void* h_params = nullptr; size_t h_params_bytes = 0;
+  void* h_obs = nullptr; size_t h_obs_bytes = 0;
+  void* h_loss = nullptr; size_t h_loss_bytes = 0;
+  void* h_grad = nullptr; size_t h_grad_bytes = 0;
+  void* h_ws = nullptr; size_t h_ws_bytes = 0;
+};
+
+}  // namespace
+
+struct ndvm_tape {
+  Tape tape;
+  Plan grad_plan, value_plan;
+  std::mutex mu;
+  std::map<int, DevCache> dev;
+};
+
+namespace {
+
+void free_plan(DevPlan& p) {
+  cudaFree(p.code); cudaFree(p.args); cudaFree(p.consts_d); cudaFree(p.consts_f);
+  p = DevPlan{};
+}
+
+ndvm_status upload_plan(const Tape& t, const Plan& p, DevPlan& d) {
+  std::vector<double> c = t.consts;
+  c.insert(c.end(), p.extra_consts.begin(), p.extra_consts.end());
+  if (c.empty()) c.push_back(0.0);
+  std::vector<float> cf(c.begin(), c.end());
+  std::vector<int32_t> args = p.args;
+  if (args.empty()) args.push_back(0);
+  cudaError_t e;
+  if ((e = cudaMalloc(&d.code, sizeof(DInst) * (p.code.size() ? p.code.size() : 1))) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+  if ((e = cudaMalloc(&d.args, sizeof(int32_t) * args.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+  if ((e = cudaMalloc(&d.consts_d, sizeof(double) * c.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+  if ((e = cudaMalloc(&d.consts_f, sizeof(float) * cf.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+  if (!p.code.empty() && (e = cudaMemcpy(d.code, p.code.data(), sizeof(DInst) * p.code.size(), cudaMemcpyHostToDevice)) != cudaSuccess)
+    return cuda_fail(e, "cudaMemcpy");
+  if ((e = cudaMemcpy(d.args, args.data(), sizeof(int32_t) * args.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  if ((e = cudaMemcpy(d.consts_d, c.data(), sizeof(double) * c.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  if ((e = cudaMemcpy(d.consts_f, cf.data(), sizeof(float) * cf.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
+  return NDVM_OK;
+}
+
+// device cache for the current device (uploads on first use)
+ndvm_status device_cache(ndvm_tape* t, DevCache** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  std::lock_guard<std::mutex> lk(t->mu);
+  auto it = t->dev.find(dev);
+  if (it == t->dev.end()) {
+    DevCache c;
+    ndvm_status s = upload_plan(t->tape, t->grad_plan, c.grad);
+    if (s == NDVM_OK) s = upload_plan(t->tape, t->value_plan, c.value);
+    if (s == NDVM_OK) {
+      if ((e = cudaMalloc(&c.err, sizeof(int))) != cudaSuccess) s = cuda_fail(e, "cudaMalloc");
+      else if ((e = cudaMemset(c.err, 0, sizeof(int))) != cudaSuccess) s = cuda_fail(e, "cudaMemset");
+    }
+    if (s != NDVM_OK) {
+      free_plan(c.grad); free_plan(c.value); cudaFree(c.err);
+      return s;
+    }
+    it = t->dev.emplace(dev, c).first;
+  }
+  *out = &it->second;
+  return NDVM_OK;
+}
+
+constexpr size_t kSmemLimit = 227 * 1024;
+
+// threads per block and threads per lane for a plan
+void launch_shape(const Plan& p, size_t elem, int64_t B, int& tpb, int& log2g) {
+  log2g = 0;
+  if (p.has_regions && p.n_save == 0) {
+    // split the data axis over a group of threads when lanes alone cannot fill the GPU
+    const int64_t target = 152LL * 1024;
+    int g = 1;
+    while (g < 32 && B * g < target) g *= 2;
+    while ((1 << log2g) < g) log2g++;
+  }
+  tpb = 128;
+  while (tpb > 32 && (size_t)p.n_slots * tpb * elem > kSmemLimit) tpb /= 2;
+}
+
+ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
+                int64_t n_obs, void* loss, void* gradp, void* ws, size_t ws_bytes, void* stream) {
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  if (dtype != NDVM_F64 && dtype != NDVM_F32) return fail(NDVM_E_INVALID_ARG, "bad dtype");
+  if (B < 0) return fail(NDVM_E_INVALID_ARG, "B must be >= 0");
+  if (B == 0) return NDVM_OK;
+  const Plan& p = grad ? t->grad_plan : t->value_plan;
+  if (B > (int64_t)1 << 40) return fail(NDVM_E_INVALID_ARG, "B too large");
+  if (p.n_params > 0 && !params) return fail(NDVM_E_INVALID_ARG, "null params");
+  if (!loss) return fail(NDVM_E_INVALID_ARG, "null loss");
+  if (grad && p.n_params > 0 && !gradp) return fail(NDVM_E_INVALID_ARG, "null grad");
+  if (n_obs < p.n_obs_min) return fail(NDVM_E_INVALID_ARG, "obs holds " + std::to_string(n_obs) + " values but the program reads " + std::to_string(p.n_obs_min));
+  if (p.n_obs_min > 0 && !obs) return fail(NDVM_E_INVALID_ARG, "null obs");
+  const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  int tpb, log2g;
+  launch_shape(p, elem, B, tpb, log2g);
+  const size_t smem = (size_t)p.n_slots * tpb * elem;
+  if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs " + std::to_string(p.n_slots) + " slots per lane, more than shared memory holds");
+  const int lanes_per_block = tpb >> log2g;
+  int64_t chunk = B;
+  if (grad && p.n_save > 0) {
+    const size_t per_lane = (size_t)p.n_save * elem;
+    if (!ws) return fail(NDVM_E_INVALID_ARG, "this tape needs a workspace of " + std::to_string(per_lane) + " bytes per lane");
+    int64_t fit = (int64_t)(ws_bytes / per_lane);
+    if (fit < B) {
+      fit -= fit % lanes_per_block;
+      if (fit < lanes_per_block)
+        return fail(NDVM_E_INVALID_ARG, "workspace too small: need at least " + std::to_string(per_lane * lanes_per_block) + " bytes");
+      chunk = fit;
+    }
+  }
+  DevCache* dc = nullptr;
+  ndvm_status s = device_cache(t, &dc);
+  if (s != NDVM_OK) return s;
+  const DevPlan& dp = grad ? dc->grad : dc->value;
+  ReplayArgs a;
+  a.code = dp.code;
+  a.n_code = (int)p.code.size();
+  a.args = dp.args;
+  a.consts = dtype == NDVM_F32 ? (const void*)dp.consts_f : (const void*)dp.consts_d;
+  a.obs = obs;
+  a.params = params;
+  a.loss = loss;
+  a.grad = gradp;
+  a.save = ws;
+  a.save_ld = chunk;
+  a.P = p.n_params;
+  a.log2g = log2g;
+  a.err = dc->err;
+  for (int64_t l0 = 0; l0 < B; l0 += chunk) {
+    a.lane0 = l0;
+    a.lane_end = l0 + chunk < B ? l0 + chunk : B;
+    const int64_t lanes = a.lane_end - l0;
+    const int64_t blocks = (lanes + lanes_per_block - 1) / lanes_per_block;
+    if (blocks > 0x7fffffff) return fail(NDVM_E_INVALID_ARG, "too many lanes for one launch");
+    cudaError_t e;
+    {
+      std::lock_guard<std::mutex> lk(g_launch_mu);
+      e = launch_replay(a, dtype == NDVM_F32, (int)blocks, tpb, smem, (cudaStream_t)stream);
+      g_launches++;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "replay launch");
+  }
+  return NDVM_OK;
+}
+
+ndvm_status ensure(void** buf, size_t* have, size_t need) {
+  if (*have >= need && *buf) return NDVM_OK;
+  cudaFree(*buf);
+  *buf = nullptr;
+  *have = 0;
+  cudaError_t e = cudaMalloc(buf, need ? need : 16);
+  if (e != cudaSuccess) return e == cudaErrorMemoryAllocation ? fail(NDVM_E_OOM, "device allocation failed") : cuda_fail(e, "cudaMalloc");
+  *have = need;
+  return NDVM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ndvm_status ndvm_trace_build(const char* program, size_t len, ndvm_frontend fe, ndvm_tape** out) {
+  if (!program || !out) return fail(NDVM_E_INVALID_ARG, "null argument");
+  if (fe != NDVM_FE_SCHEME && fe != NDVM_FE_BYTECODE) return fail(NDVM_E_INVALID_ARG, "unknown front end");
+  *out = nullptr;
+  try {
+    Builder b;
+    std::string err;
+    if (fe == NDVM_FE_SCHEME) trace_scheme(program, len, b, err);
+    else trace_bytecode(program, len, b, err);
+    if (b.t.loss < 0) return fail(NDVM_E_PARSE, "program produced no result");
+    ndvm_tape* t = new ndvm_tape();
+    t->tape = std::move(b.t);
+    t->grad_plan = make_plan(t->tape, true);
+    t->value_plan = make_plan(t->tape, false);
+    std::string why;
+    if (!validate_plan(t->grad_plan, t->tape.consts.size(), why) || !validate_plan(t->value_plan, t->tape.consts.size(), why)) {
+      delete t;
+      return fail(NDVM_E_UNSUPPORTED, "internal plan check failed: " + why);
+    }
+    *out = t;
+    return NDVM_OK;
+  } catch (const BuildError& e) {
+    return fail((ndvm_status)e.code, e.msg);
+  } catch (const std::bad_alloc&) {
+    return fail(NDVM_E_OOM, "host allocation failed");
+  } catch (const std::exception& e) {
+    return fail(NDVM_E_UNSUPPORTED, e.what());
+  }
+}
+
+ndvm_status ndvm_tape_info(const ndvm_tape* t, int64_t* n_nodes, int32_t* n_params, int64_t* n_obs, int64_t* n_slots,
+                           uint64_t* hash) {
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  if (n_nodes) *n_nodes = (int64_t)t->tape.nodes.size();
+  if (n_params) *n_params = t->tape.n_params;
+  if (n_obs) *n_obs = t->tape.n_obs_min;
+  if (n_slots) *n_slots = t->grad_plan.n_slots;
+  if (hash) *hash = t->tape.hash();
+  return NDVM_OK;
+}
+
+ndvm_status ndvm_tape_cost(const ndvm_tape* t, double* work_fwd, double* work_rev, int64_t* save_elems,
+                           int32_t* flags) {
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  const Plan& p = t->grad_plan;
+  if (work_fwd) *work_fwd = p.work_fwd;
+  if (work_rev) *work_rev = p.work_rev;
+  if (save_elems) *save_elems = p.n_save;
+  if (flags) *flags = (p.has_regions ? 1 : 0) | (p.spill ? 2 : 0);
+  return NDVM_OK;
+}
+
+ndvm_status ndvm_tape_serialize(const ndvm_tape* t, void* buf, size_t cap, size_t* len) {
+  if (!t || !len) return fail(NDVM_E_INVALID_ARG, "null argument");
+  std::vector<uint8_t> s = t->tape.serialize();
+  *len = s.size();
+  if (!buf && cap == 0) return NDVM_OK;
+  if (!buf || cap < s.size()) return fail(NDVM_E_INVALID_ARG, "buffer too small");
+  std::memcpy(buf, s.data(), s.size());
+  return NDVM_OK;
+}
+
+void ndvm_tape_free(ndvm_tape* t) {
+  if (!t) return;
+  int cur = 0;
+  cudaGetDevice(&cur);
+  for (auto& kv : t->dev) {
+    cudaSetDevice(kv.first);
+    DevCache& c = kv.second;
+    free_plan(c.grad); free_plan(c.value);
+    cudaFree(c.err);
+    cudaFree(c.h_params); cudaFree(c.h_obs); cudaFree(c.h_loss); cudaFree(c.h_grad); cudaFree(c.h_ws);
+  }
+  if (!t->dev.empty()) cudaSetDevice(cur);
+  delete t;
+}
+
+size_t ndvm_workspace_bytes(const ndvm_tape* t, int64_t B, ndvm_dtype dtype) {
+  if (!t || B <= 0) return 0;
+  size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  return (size_t)t->grad_plan.n_save * elem * (size_t)B;
+}
+
+ndvm_status ndvm_forward(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
+                         int64_t n_obs, void* loss, void* stream) {
+  return run(const_cast<ndvm_tape*>(tape), false, dtype, B, params, obs, n_obs, loss, nullptr, nullptr, 0, stream);
+}
+
+ndvm_status ndvm_value_and_grad(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                const void* obs, int64_t n_obs, void* loss, void* grad, void* ws, size_t ws_bytes,
+                                void* stream) {
+  return run(const_cast<ndvm_tape*>(tape), true, dtype, B, params, obs, n_obs, loss, grad, ws, ws_bytes, stream);
+}
+
+ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                     const void* obs, int64_t n_obs, void* loss, void* grad, void* stream) {
+  ndvm_tape* t = const_cast<ndvm_tape*>(tape);
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  if (B < 0 || n_obs < 0) return fail(NDVM_E_INVALID_ARG, "negative size");
+  if (B == 0) return NDVM_OK;
+  if (!loss || (t->tape.n_params > 0 && !params) || (n_obs > 0 && !obs)) return fail(NDVM_E_INVALID_ARG, "null argument");
+  DevCache* dc = nullptr;
+  ndvm_status s = device_cache(t, &dc);
+  if (s != NDVM_OK) return s;
+  const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  const size_t pb = (size_t)B * t->tape.n_params * elem, ob = (size_t)n_obs * elem, lb = (size_t)B * elem;
+  const bool want_grad = grad != nullptr;
+  size_t wsb = want_grad ? ndvm_workspace_bytes(t, B, dtype) : 0;
+  std::lock_guard<std::mutex> lk(t->mu);
+  if ((s = ensure(&dc->h_params, &dc->h_params_bytes, pb)) != NDVM_OK) return s;
+  if ((s = ensure(&dc->h_obs, &dc->h_obs_bytes, ob)) != NDVM_OK) return s;
+  if ((s = ensure(&dc->h_loss, &dc->h_loss_bytes, lb)) != NDVM_OK) return s;
+  if (want_grad && (s = ensure(&dc->h_grad, &dc->h_grad_bytes, pb)) != NDVM_OK) return s;
+  if (wsb && (s = ensure(&dc->h_ws, &dc->h_ws_bytes, wsb)) != NDVM_OK) return s;
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e;
+  if (pb && (e = cudaMemcpyAsync(dc->h_params, params, pb, cudaMemcpyHostToDevice, st)) != cudaSuccess) return cuda_fail(e, "copy params");
+  if (ob && (e = cudaMemcpyAsync(dc->h_obs, obs, ob, cudaMemcpyHostToDevice, st)) != cudaSuccess) return cuda_fail(e, "copy obs");
+  if (want_grad)
+    s = run(t, true, dtype, B, dc->h_params, n_obs ? dc->h_obs : nullptr, n_obs, dc->h_loss, dc->h_grad, dc->h_ws, wsb, stream);
+  else
+    s = run(t, false, dtype, B, dc->h_params, n_obs ? dc->h_obs : nullptr, n_obs, dc->h_loss, nullptr, nullptr, 0, stream);
+  if (s != NDVM_OK) return s;
+  if ((e = cudaMemcpyAsync(loss, dc->h_loss, lb, cudaMemcpyDeviceToHost, st)) != cudaSuccess) return cuda_fail(e, "copy loss");
+  if (want_grad && pb && (e = cudaMemcpyAsync(grad, dc->h_grad, pb, cudaMemcpyDeviceToHost, st)) != cudaSuccess) return cuda_fail(e, "copy grad");
+  if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return cuda_fail(e, "synchronize");
+  return NDVM_OK;
+}
+
+ndvm_status ndvm_check_device(const ndvm_tape* tape) {
+  ndvm_tape* t = const_cast<ndvm_tape*>(tape);
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  DevCache* dc = nullptr;
+  ndvm_status s = device_cache(t, &dc);
+  if (s != NDVM_OK) return s;
+  int flag = 0;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "synchronize");
+  if ((e = cudaMemcpy(&flag, dc->err, sizeof(int), cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "read flag");
+  if (flag) {
+    cudaMemset(dc->err, 0, sizeof(int));
+    return fail(NDVM_E_DEVICE_CHECK, "a replay kernel met an invalid instruction");
+  }
+  return NDVM_OK;
+}
+
+ndvm_status ndvm_measure_fp64_peak(double* flops_per_s, void* stream) {
+  if (!flops_per_s) return fail(NDVM_E_INVALID_ARG, "null output");
+  cudaError_t e = measure_fp64_peak(flops_per_s, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "fp64 peak probe");
+  return NDVM_OK;
+}
+
+unsigned long long ndvm_launch_count(void) {
+  std::lock_guard<std::mutex> lk(g_launch_mu);
+  return g_launches;
+}
+
+const char* ndvm_last_error(void) { return g_last_error.c_str(); }
+
+const char* ndvm_version(void) { return "ndvm-gb300 0.1"; }
+
+}  // extern "C"

@@ -1,0 +1,87 @@
+// Algorithmic FP64 work per tape primitive, in DFMA-equivalents (one fused
+// multiply-add issue of the FP64 pipe = 1).  Arithmetic counts one per add,
+// multiply or fused multiply-add; a first adjoint contribution that is a copy or a
+// sign flip counts zero.  Library functions count their throughput cost relative
+// to DFMA, measured on GB300 for CUDA's double-precision functions with many
+// independent calls per thread (exp 17.6, log 28.7, sin or cos 17.4, sincos 22.7,
+// tanh 13.7, sqrt 7.5, reciprocal 4.6, pow 85).  The roofline divides this work by
+// the measured DFMA rate.
+#pragma once
+#include "tape.h"
+
+namespace ndvm {
+namespace cost {
+
+constexpr double kExp = 17.6, kLog = 28.7, kSin = 17.4, kSinCos = 22.7, kTanh = 13.7, kSqrt = 7.5,
+                 kRcp = 4.6, kPow = 85.0;
+constexpr double kDiv = kRcp + 1.0;
+
+inline double inv_cost(int n) {
+  if (n == 1) return kDiv;
+  if (n == 2) return 2 + kDiv + 4;           // det, 1/det, four scaled cofactors
+  if (n == 3) return 18 + 3 + kDiv + 9;      // nine cofactors, det, 1/det, nine scalings
+  return 2.0 * n * n * n + n * kDiv;        // elimination
+}
+inline double det_cost(int n) {
+  if (n == 1) return 0;
+  if (n == 2) return 2;
+  if (n == 3) return 9;
+  return (2.0 * n * n * n) / 3.0 + n * kDiv;
+}
+
+inline double fwd(int op, int r, int c, int imm, int n, bool with_aux) {
+  const double e = (double)r * c;
+  switch (op) {
+    case OP_ADD: case OP_SUB: case OP_MUL: return 1;
+    case OP_DIV: return kDiv;
+    case OP_POW: return kPow;
+    case OP_NEG: case OP_ABS: case OP_SELECT: return 0;
+    case OP_EXP: return kExp;
+    case OP_LOG: return kLog;
+    case OP_SIN: case OP_COS: return with_aux ? kSinCos : kSin;
+    case OP_TANH: return kTanh;
+    case OP_SQRT: return kSqrt;
+    case OP_POWI: return imm > 1 ? imm - 1 : 0;
+    case OP_LT: case OP_LE: case OP_GT: case OP_GE: case OP_EQ: return 1;
+    case OP_MADD: case OP_MSUB: case OP_MSCALE: return e;
+    case OP_MATMUL: return e * imm;
+    case OP_INV: return inv_cost(n);
+    case OP_DET: return with_aux ? inv_cost(n) : det_cost(n);
+    case OP_LOGDET: return (with_aux ? inv_cost(n) : det_cost(n)) + kLog;
+    case OP_TRACE: return n - 1;
+    default: return 0;
+  }
+}
+
+// a_init / b_init: the contribution is the first one to that input's adjoint
+inline double rev(int op, int r, int c, int imm, int n, bool aa, bool ba, bool a_init, bool b_init, int extra) {
+  const double e = (double)r * c;
+  auto acc = [](bool active, bool init) { return active && !init ? 1.0 : 0.0; };
+  switch (op) {
+    case OP_ADD: case OP_SUB: return acc(aa, a_init) + acc(ba, b_init);
+    case OP_NEG: return acc(aa, a_init);
+    case OP_MUL: return (aa ? 1 : 0) + (ba ? 1 : 0);
+    case OP_DIV: return kDiv + acc(aa, a_init) + (ba ? 1 : 0);
+    case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLog + 2 : 0);
+    case OP_EXP: case OP_SIN: case OP_COS: case OP_ABS: return 1;
+    case OP_TANH: return 2;
+    case OP_LOG: return kDiv + 1;
+    case OP_SQRT: return kDiv + 2;
+    case OP_POWI: return imm > 0 ? imm : 0;
+    case OP_SELECT: return acc(aa, a_init) + acc(ba, b_init);
+    case OP_MATFROM: return 0.0 + extra * 0.5;  // scattered copies and adds
+    case OP_MREF: case OP_SUBMAT: case OP_TRANSPOSE: return a_init ? 0 : e;
+    case OP_MADD: case OP_MSUB: return (aa && !a_init ? e : 0) + (ba && !b_init ? e : 0);
+    case OP_MSCALE: return (aa ? e : 0) + (ba ? e : 0);
+    case OP_MATMUL: return (aa ? e * imm : 0) + (ba ? e * imm : 0);
+    case OP_INV: return 2.0 * n * n * n;
+    case OP_DET: return 2.0 * n * n;
+    case OP_LOGDET: return 1.0 * n * n;
+    case OP_TRACE: return a_init ? 0 : n;
+    case OP_DSUM: return 2.0 * extra;
+    default: return 0;
+  }
+}
+
+}  // namespace cost
+}  // namespace ndvm

@@ -1,0 +1,776 @@
+// Planner: lowers a Tape (SSA, section 3.4) to the device instruction stream.
+//
+// Forward sweep: one instruction per non-leaf node, in tape order.  A data-axis
+// region (section 3.5) becomes a loop over the lane's data points whose body runs
+// the region's forward instructions, then immediately its reverse instructions
+// seeded with d(body)/d(body) = 1, accumulating the body value and the partial
+// derivatives of the body with respect to its lane-level inputs.  Because the
+// region's output is a sum, the adjoint of each region input is later
+// g_sum * (sum over points of its partial) -- exact by linearity.
+// Reverse sweep: one instruction per active node in reverse tape order, using
+// the adjoint rules of Appendix C (and readings for tanh/neg/select/compare).
+#include "plan.h"
+
+#include <algorithm>
+#include <climits>
+#include <cstring>
+#include <set>
+
+#include "cost.h"
+#include "status.h"
+
+namespace ndvm {
+namespace {
+
+[[noreturn]] void unsupported(const std::string& m) { throw BuildError{NDVM_E_UNSUPPORTED, m}; }
+
+struct PRef {
+  uint32_t kind = RK_SLOT;
+  int32_t id = -1;  // VR id for slots; index otherwise
+  int32_t off = 0;
+};
+struct PArg {
+  bool isref = false;
+  PRef r;
+  int32_t v = -1;
+};
+inline PArg I(int32_t v) { PArg a; a.v = v; return a; }
+inline PArg R(PRef r) { PArg a; a.isref = true; a.r = r; return a; }
+inline PRef slotref(int vr, int off = 0) { PRef r; r.kind = RK_SLOT; r.id = vr; r.off = off; return r; }
+inline PRef kref(uint32_t kind, int32_t idx) { PRef r; r.kind = kind; r.id = idx; return r; }
+
+struct PInst {
+  DInst d;
+  PArg f[8];
+};
+
+struct VR {
+  int width;
+  int start = INT_MAX, end = -1, phys = -1;
+};
+
+class Planner {
+ public:
+  Planner(const Tape& t, bool grad, bool spill) : T(t), grad_(grad), spill_(spill) {}
+  Plan build();
+
+ private:
+  const Tape& T;
+  bool grad_, spill_;
+  int N = 0;
+  std::vector<uint8_t> active_, region_body_;
+  std::vector<char> need_val_, need_aux_;
+  std::vector<int> val_vr_, aux_vr_, adj_vr_;
+  std::vector<int64_t> save_, aux_save_;
+  std::vector<VR> vrs_;
+  std::vector<PInst> code_;
+  std::vector<PArg> args_;
+  int64_t S_ = 0;
+  double work_fwd_ = 0, work_rev_ = 0, nops_ = 0;
+  // data-axis regions
+  int cur_region_ = -1;          // DSUM node whose body is being emitted
+  std::vector<int> partial_of_;  // node -> offset of its partial in the block (current region)
+  int block_vr_ = -1;            // current region: [sum, partials...]
+  std::vector<int> body_adj_;    // node -> adjoint VR inside the current region body
+  std::vector<std::vector<std::pair<int, int>>> region_inputs_;  // DSUM node -> (input, offset)
+  std::vector<int> region_block_;                                // DSUM node -> block VR
+  int one_const_ = -1;
+  double mult_ = 1.0;  // executions per lane of the instruction being emitted
+  std::vector<double> extra_consts_;
+  int n_slots_ = 0;
+
+  int width(int v) const { return T.nodes[v].rows * T.nodes[v].cols; }
+  bool is_leaf(int v) const {
+    uint16_t op = T.nodes[v].op;
+    return op == OP_CONST || op == OP_PARAM || op == OP_OBS || op == OP_DOBS;
+  }
+  int new_vr(int w) { vrs_.push_back(VR{w}); return (int)vrs_.size() - 1; }
+  int emit(const PInst& p) { code_.push_back(p); return (int)code_.size() - 1; }
+
+  std::vector<int> inputs(int v) const;
+  void analyze();
+  PRef ref(int v);          // primal reference for forward use
+  PRef rref(int v);         // primal reference for reverse use
+  PRef rauxref(int v);
+  PArg save_of(int v) { return I(spill_ && save_[v] >= 0 ? (int32_t)save_[v] : -1); }
+  void emit_forward(int v);
+  void emit_region(int v);
+  // adjoint target of input x during reverse: returns (slot ref, first-contribution flag)
+  std::pair<PRef, bool> target(int x);
+  void emit_reverse(int v);
+  void allocate();
+  int32_t encode(const PArg& a) const;
+};
+
+std::vector<int> Planner::inputs(int v) const {
+  const Node& n = T.nodes[v];
+  std::vector<int> r;
+  switch (n.op) {
+    case OP_CONST: case OP_PARAM: case OP_OBS: case OP_DOBS: break;
+    case OP_MATFROM: for (int k = 0; k < n.rows * n.cols; k++) r.push_back(T.args[n.imm + k]); break;
+    case OP_SELECT: r = {n.a, n.b, n.c}; break;
+    case OP_DSUM: r = {n.c}; break;
+    default:
+      if (n.a >= 0) r.push_back(n.a);
+      if (n.b >= 0) r.push_back(n.b);
+      break;
+  }
+  return r;
+}
+
+void Planner::analyze() {
+  N = (int)T.nodes.size();
+  active_.assign(N, 0);
+  region_body_.assign(N, 0);
+  for (int v = 0; v < N; v++) {
+    const Node& n = T.nodes[v];
+    if (n.op == OP_DSUM) {
+      for (int u = n.a; u < n.b; u++) region_body_[u] = 1;
+      if (n.c >= n.a && n.c < n.b) {} else if (n.c >= v) unsupported("malformed data-sum");
+    }
+  }
+  for (int v = 0; v < N; v++) {
+    const Node& n = T.nodes[v];
+    switch (n.op) {
+      case OP_PARAM: active_[v] = 1; break;
+      case OP_CONST: case OP_OBS: case OP_DOBS: break;
+      case OP_LT: case OP_LE: case OP_GT: case OP_GE: case OP_EQ: break;  // no gradient through a test
+      case OP_SELECT: active_[v] = active_[n.b] || active_[n.c]; break;
+      default:
+        for (int x : inputs(v)) {
+          if (x < 0 || x >= v) unsupported("tape is not in SSA order");
+          if (active_[x]) active_[v] = 1;
+        }
+    }
+    // body values must not escape their region (leaves are shared)
+    if (!region_body_[v] || n.op == OP_DSUM) {
+      for (int x : inputs(v))
+        if (region_body_[x] && !is_leaf(x) && n.op != OP_DSUM) unsupported("a data-sum body value escapes its region");
+    }
+  }
+  need_val_.assign(N, 0);
+  need_aux_.assign(N, 0);
+  if (grad_) {
+    for (int v = 0; v < N; v++) {
+      if (!active_[v]) continue;
+      const Node& n = T.nodes[v];
+      auto need = [&](int x) { need_val_[x] = 1; };
+      switch (n.op) {
+        case OP_MUL: if (active_[n.a]) need(n.b); if (active_[n.b]) need(n.a); break;
+        case OP_DIV: if (active_[n.a]) need(n.b); if (active_[n.b]) { need(n.b); need(v); } break;
+        case OP_POW: need(n.a); need(n.b); need(v); break;
+        case OP_EXP: case OP_TANH: case OP_INV: need(v); break;
+        case OP_LOG: case OP_ABS: case OP_POWI: need(n.a); break;
+        case OP_SQRT: need(n.a); need(v); break;
+        case OP_SIN: case OP_COS: need_aux_[v] = 1; break;
+        case OP_SELECT: need(n.a); break;
+        case OP_MSCALE: if (active_[n.a]) need(n.b); if (active_[n.b]) need(n.a); break;
+        case OP_MATMUL: if (active_[n.a]) need(n.b); if (active_[n.b]) need(n.a); break;
+        case OP_DET: need(v); need_aux_[v] = 1; break;
+        case OP_LOGDET: need_aux_[v] = 1; break;
+        default: break;
+      }
+    }
+  }
+  val_vr_.assign(N, -1);
+  aux_vr_.assign(N, -1);
+  adj_vr_.assign(N, -1);
+  save_.assign(N, -1);
+  aux_save_.assign(N, -1);
+  body_adj_.assign(N, -1);
+  partial_of_.assign(N, -1);
+  region_inputs_.assign(N, {});
+  region_block_.assign(N, -1);
+  for (int v = 0; v < N; v++) {
+    if (is_leaf(v) || T.nodes[v].op == OP_DSUM) continue;
+    val_vr_[v] = new_vr(width(v));
+    bool lane_level = !region_body_[v];
+    if (need_aux_[v]) {
+      int aw = (T.nodes[v].op == OP_DET || T.nodes[v].op == OP_LOGDET) ? width(T.nodes[v].a) : 1;
+      if (spill_ && lane_level) { aux_save_[v] = S_; S_ += aw; }
+      else aux_vr_[v] = new_vr(aw);
+    }
+    if (spill_ && lane_level && need_val_[v]) { save_[v] = S_; S_ += width(v); }
+  }
+}
+
+PRef Planner::ref(int v) {
+  const Node& n = T.nodes[v];
+  switch (n.op) {
+    case OP_CONST: return kref(RK_CONST, n.imm);
+    case OP_PARAM: return kref(RK_PARAM, n.imm);
+    case OP_OBS: return kref(RK_OBS, n.imm);
+    case OP_DOBS: return kref(RK_DOBS, n.imm);
+    case OP_DSUM: return slotref(val_vr_[v], 0);
+    default: return slotref(val_vr_[v]);
+  }
+}
+
+PRef Planner::rref(int v) {
+  if (!is_leaf(v) && T.nodes[v].op != OP_DSUM && spill_ && !region_body_[v]) {
+    if (save_[v] < 0) unsupported("internal: reverse reads an unsaved value");
+    return kref(RK_SAVE, (int32_t)save_[v]);
+  }
+  return ref(v);
+}
+
+PRef Planner::rauxref(int v) {
+  if (spill_ && !region_body_[v]) return kref(RK_SAVE, (int32_t)aux_save_[v]);
+  return slotref(aux_vr_[v]);
+}
+
+void Planner::emit_forward(int v) {
+  const Node& n = T.nodes[v];
+  PInst p;
+  p.d.r = n.rows; p.d.c = n.cols;
+  PRef out = slotref(val_vr_[v]);
+  p.f[0] = R(out);
+  work_fwd_ += mult_ * cost::fwd(n.op, n.rows, n.cols, n.imm, T.nodes[n.a >= 0 ? n.a : v].rows, grad_ && need_aux_[v]);
+  nops_ += mult_;
+  switch (n.op) {
+    case OP_ADD: case OP_SUB: case OP_MUL: case OP_DIV: case OP_POW:
+      p.d.op = n.op == OP_ADD ? D_ADD : n.op == OP_SUB ? D_SUB : n.op == OP_MUL ? D_MUL : n.op == OP_DIV ? D_DIV : D_POW;
+      p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      break;
+    case OP_NEG: case OP_EXP: case OP_LOG: case OP_TANH: case OP_SQRT: case OP_ABS:
+      p.d.op = n.op == OP_NEG ? D_NEG : n.op == OP_EXP ? D_EXP : n.op == OP_LOG ? D_LOG : n.op == OP_TANH ? D_TANH
+             : n.op == OP_SQRT ? D_SQRT : D_ABS;
+      p.f[1] = R(ref(n.a)); p.f[3] = save_of(v);
+      break;
+    case OP_SIN: case OP_COS:
+      p.d.op = n.op == OP_SIN ? D_SIN : D_COS;
+      p.f[1] = R(ref(n.a)); p.f[3] = save_of(v);
+      if (need_aux_[v]) {
+        if (aux_vr_[v] >= 0) p.f[4] = R(slotref(aux_vr_[v]));
+        else p.f[5] = I((int32_t)aux_save_[v]);
+      }
+      break;
+    case OP_POWI:
+      p.d.op = D_POWI; p.f[1] = R(ref(n.a)); p.f[3] = save_of(v); p.f[7] = I(n.imm);
+      break;
+    case OP_LT: case OP_LE: case OP_GT: case OP_GE: case OP_EQ:
+      p.d.op = D_CMP;
+      p.d.k = n.op == OP_LT ? 0 : n.op == OP_LE ? 1 : n.op == OP_GT ? 2 : n.op == OP_GE ? 3 : 4;
+      p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      break;
+    case OP_SELECT:
+      p.d.op = D_SELECT; p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[4] = R(ref(n.c)); p.f[3] = save_of(v);
+      break;
+    case OP_MATFROM: {
+      p.d.op = D_GATHER;
+      p.f[1] = I((int32_t)args_.size()); p.f[2] = I(n.rows * n.cols); p.f[3] = save_of(v);
+      for (int k = 0; k < n.rows * n.cols; k++) args_.push_back(R(ref(T.args[n.imm + k])));
+      break;
+    }
+    case OP_MREF: case OP_SUBMAT: case OP_TRANSPOSE: {
+      // pure data movement: a gather of input elements
+      p.d.op = D_GATHER;
+      const Node& in = T.nodes[n.a];
+      PRef base = ref(n.a);
+      p.f[1] = I((int32_t)args_.size()); p.f[2] = I(n.rows * n.cols); p.f[3] = save_of(v);
+      for (int i = 0; i < n.rows; i++)
+        for (int j = 0; j < n.cols; j++) {
+          int e;
+          if (n.op == OP_MREF) e = n.imm;
+          else if (n.op == OP_SUBMAT) e = (n.imm + i) * in.cols + n.imm2 + j;
+          else e = j * in.cols + i;  // transpose: out(i,j) = in(j,i)
+          PRef r = base; r.off += e;
+          args_.push_back(R(r));
+        }
+      break;
+    }
+    case OP_MADD: case OP_MSUB:
+      p.d.op = n.op == OP_MADD ? D_MADD : D_MSUB;
+      p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      break;
+    case OP_MSCALE:
+      p.d.op = D_MSCALE; p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      break;
+    case OP_MATMUL:
+      p.d.op = D_MATMUL; p.d.k = (uint8_t)n.imm;
+      p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      break;
+    case OP_INV:
+      p.d.op = D_INV; p.d.r = T.nodes[n.a].rows; p.f[1] = R(ref(n.a)); p.f[3] = save_of(v);
+      break;
+    case OP_DET: case OP_LOGDET:
+      p.d.op = n.op == OP_DET ? D_DET : D_LOGDET; p.d.r = T.nodes[n.a].rows; p.d.c = 1;
+      p.f[1] = R(ref(n.a)); p.f[3] = save_of(v);
+      if (need_aux_[v]) {
+        if (aux_vr_[v] >= 0) p.f[4] = R(slotref(aux_vr_[v]));
+        else p.f[5] = I((int32_t)aux_save_[v]);
+      }
+      break;
+    case OP_TRACE:
+      p.d.op = D_TRACE; p.d.r = T.nodes[n.a].rows; p.d.c = 1; p.f[1] = R(ref(n.a));
+      break;
+    default:
+      unsupported(std::string("no forward lowering for ") + op_name(n.op));
+  }
+  emit(p);
+}
+
+std::pair<PRef, bool> Planner::target(int x) {
+  // inside a region body: body values get body adjoints, lane values get partial slots
+  if (cur_region_ >= 0) {
+    if (region_body_[x] && !is_leaf(x)) {
+      if (body_adj_[x] < 0) { body_adj_[x] = new_vr(width(x)); return {slotref(body_adj_[x]), true}; }
+      return {slotref(body_adj_[x]), false};
+    }
+    if (partial_of_[x] < 0) unsupported("internal: region input without a partial slot");
+    return {slotref(block_vr_, partial_of_[x]), false};
+  }
+  if (adj_vr_[x] < 0) { adj_vr_[x] = new_vr(width(x)); return {slotref(adj_vr_[x]), true}; }
+  return {slotref(adj_vr_[x]), false};
+}
+
+void Planner::emit_reverse(int v) {
+  const Node& n = T.nodes[v];
+  int gz_vr = cur_region_ >= 0 ? body_adj_[v] : adj_vr_[v];
+  if (gz_vr < 0) return;  // no contribution reached this node: its adjoint is zero
+  PInst p;
+  p.d.r = n.rows; p.d.c = n.cols;
+  p.f[0] = R(slotref(gz_vr));
+  uint8_t flags = 0;
+  auto tgt = [&](int x, int field, int bit) {
+    if (!active_[x]) return;
+    auto t = target(x);
+    p.f[field] = R(t.first);
+    if (t.second) flags |= (uint8_t)(1u << bit);
+  };
+  switch (n.op) {
+    case OP_ADD: case OP_SUB:
+      p.d.op = n.op == OP_ADD ? B_ADD : B_SUB; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      break;
+    case OP_MUL:
+      p.d.op = B_MUL; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      if (active_[n.a]) p.f[4] = R(rref(n.b));
+      if (active_[n.b]) p.f[3] = R(rref(n.a));
+      break;
+    case OP_DIV:
+      p.d.op = B_DIV; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      p.f[4] = R(rref(n.b));
+      if (active_[n.b]) p.f[5] = R(rref(v));
+      break;
+    case OP_POW:
+      p.d.op = B_POW; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      p.f[3] = R(rref(n.a)); p.f[4] = R(rref(n.b)); p.f[5] = R(rref(v));
+      break;
+    case OP_NEG: p.d.op = B_NEG; tgt(n.a, 1, 0); break;
+    case OP_EXP: case OP_TANH: p.d.op = n.op == OP_EXP ? B_EXP : B_TANH; tgt(n.a, 1, 0); p.f[5] = R(rref(v)); break;
+    case OP_LOG: case OP_ABS: p.d.op = n.op == OP_LOG ? B_LOG : B_ABS; tgt(n.a, 1, 0); p.f[3] = R(rref(n.a)); break;
+    case OP_SQRT: p.d.op = B_SQRT; tgt(n.a, 1, 0); p.f[3] = R(rref(n.a)); p.f[5] = R(rref(v)); break;
+    case OP_SIN: case OP_COS: p.d.op = n.op == OP_SIN ? B_SIN : B_COS; tgt(n.a, 1, 0); p.f[6] = R(rauxref(v)); break;
+    case OP_POWI: p.d.op = B_POWI; tgt(n.a, 1, 0); p.f[3] = R(rref(n.a)); p.f[7] = I(n.imm); break;
+    case OP_SELECT:
+      p.d.op = B_SELECT; tgt(n.b, 1, 0); tgt(n.c, 2, 1); p.f[3] = R(rref(n.a));
+      break;
+    case OP_MATFROM: {
+      p.d.op = B_GATHER;
+      int cnt = n.rows * n.cols;
+      p.f[1] = I((int32_t)args_.size()); p.f[2] = I(cnt);
+      for (int k = 0; k < cnt; k++) {
+        int x = T.args[n.imm + k];
+        if (!active_[x]) { args_.push_back(I(-1)); args_.push_back(I(0)); continue; }
+        auto t = target(x);
+        args_.push_back(R(t.first));
+        args_.push_back(I(t.second ? 1 : 0));
+      }
+      break;
+    }
+    case OP_MREF: case OP_SUBMAT: case OP_TRANSPOSE: {
+      p.d.op = B_SCATTER;
+      const Node& in = T.nodes[n.a];
+      tgt(n.a, 1, 0);
+      p.f[2] = I(n.rows * n.cols); p.f[3] = I((int32_t)args_.size()); p.f[4] = I(in.rows * in.cols);
+      for (int i = 0; i < n.rows; i++)
+        for (int j = 0; j < n.cols; j++) {
+          int e;
+          if (n.op == OP_MREF) e = n.imm;
+          else if (n.op == OP_SUBMAT) e = (n.imm + i) * in.cols + n.imm2 + j;
+          else e = j * in.cols + i;
+          args_.push_back(I(e));
+        }
+      break;
+    }
+    case OP_MADD: case OP_MSUB: p.d.op = n.op == OP_MADD ? B_MADD : B_MSUB; tgt(n.a, 1, 0); tgt(n.b, 2, 1); break;
+    case OP_MSCALE:
+      p.d.op = B_MSCALE; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      if (active_[n.a]) p.f[4] = R(rref(n.b));
+      if (active_[n.b]) p.f[3] = R(rref(n.a));
+      break;
+    case OP_MATMUL:
+      p.d.op = B_MATMUL; p.d.k = (uint8_t)n.imm; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
+      if (active_[n.a]) p.f[4] = R(rref(n.b));
+      if (active_[n.b]) p.f[3] = R(rref(n.a));
+      break;
+    case OP_INV: p.d.op = B_INV; p.d.r = T.nodes[n.a].rows; tgt(n.a, 1, 0); p.f[5] = R(rref(v)); break;
+    case OP_DET:
+      p.d.op = B_DET; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0);
+      p.f[5] = R(rref(v)); p.f[6] = R(rauxref(v));
+      break;
+    case OP_LOGDET: p.d.op = B_LOGDET; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0); p.f[6] = R(rauxref(v)); break;
+    case OP_TRACE: p.d.op = B_TRACE; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0); break;
+    case OP_DSUM: {
+      p.d.op = B_DSUM;
+      const auto& ins = region_inputs_[v];
+      p.f[1] = I((int32_t)args_.size()); p.f[2] = I((int32_t)ins.size());
+      for (auto& io : ins) {
+        auto t = target(io.first);
+        args_.push_back(R(t.first));
+        args_.push_back(I(t.second ? 1 : 0));
+        args_.push_back(R(slotref(region_block_[v], io.second)));
+      }
+      break;
+    }
+    default:
+      return;  // leaves and comparisons carry no adjoint
+  }
+  p.d.flags = flags;
+  {
+    int in_rows = T.nodes[n.a >= 0 ? n.a : v].rows;
+    bool aa = false, ba = false;
+    if (n.op == OP_SELECT) { aa = active_[n.b]; ba = active_[n.c]; }
+    else if (n.op != OP_MATFROM && n.op != OP_DSUM) { aa = n.a >= 0 && active_[n.a]; ba = n.b >= 0 && active_[n.b]; }
+    int extra = 0;
+    if (n.op == OP_MATFROM) for (int k = 0; k < n.rows * n.cols; k++) extra += active_[T.args[n.imm + k]] ? 1 : 0;
+    if (n.op == OP_DSUM) extra = (int)region_inputs_[v].size();
+    work_rev_ += mult_ * cost::rev(n.op, n.rows, n.cols, n.imm, in_rows, aa, ba, (flags & 1) != 0, (flags & 2) != 0, extra);
+  }
+  emit(p);
+}
+
+void Planner::emit_region(int v) {
+  const Node& n = T.nodes[v];
+  const int b0 = n.a, b1 = n.b, res = n.c;
+  auto body_value = [&](int x) { return x >= b0 && x < b1 && !is_leaf(x); };
+  // lane-level inputs whose partials the body reverse accumulates
+  std::vector<std::pair<int, int>> ins;
+  std::vector<char> seen(N, 0);
+  auto add_input = [&](int x) {
+    if (!grad_ || !active_[x] || body_value(x) || seen[x]) return;
+    seen[x] = 1;
+    ins.push_back({x, 1 + (int)ins.size()});
+  };
+  if (grad_) {
+    for (int u = b0; u < b1; u++) {
+      if (is_leaf(u) || !active_[u]) continue;
+      const Node& m = T.nodes[u];
+      if (m.op == OP_SELECT) { add_input(m.b); add_input(m.c); continue; }
+      for (int x : inputs(u)) add_input(x);
+    }
+    add_input(res);
+  }
+  int block = new_vr(1 + (int)ins.size());
+  region_inputs_[v] = ins;
+  region_block_[v] = block;
+  val_vr_[v] = block;  // the sum is element 0 of the block
+  const int32_t stride = T.args[n.imm2], base = T.args[n.imm2 + 1];
+
+  PInst z; z.d.op = D_ZERO; z.f[0] = R(slotref(block)); z.f[1] = I(1 + (int)ins.size());
+  emit(z);
+  PInst lp; lp.d.op = D_LOOP; lp.f[0] = I(n.imm); lp.f[1] = I(stride); lp.f[2] = I(base);
+  int loop_pc = emit(lp);
+  mult_ = (double)n.imm;
+  work_fwd_ += mult_;  // accumulation of the body value
+  for (int u = b0; u < b1; u++) {
+    if (is_leaf(u)) continue;
+    if (T.nodes[u].op == OP_DSUM) unsupported("nested data-sum");
+    emit_forward(u);
+  }
+  PInst acc; acc.d.op = D_ACC; acc.f[0] = R(slotref(block, 0)); acc.f[1] = R(ref(res));
+  emit(acc);
+  if (grad_ && active_[res]) {
+    cur_region_ = v;
+    block_vr_ = block;
+    for (auto& io : ins) partial_of_[io.first] = io.second;
+    if (body_value(res)) {
+      body_adj_[res] = new_vr(1);
+      PInst sd; sd.d.op = D_SEED; sd.f[0] = R(slotref(body_adj_[res]));
+      emit(sd);
+    } else {
+      // the body result is a lane-level value: d(body)/d(res) = 1 at every point
+      PInst a1; a1.d.op = D_ACC; a1.f[0] = R(slotref(block, partial_of_[res]));
+      a1.f[1] = R(kref(RK_CONST, one_const_));
+      emit(a1);
+    }
+    for (int u = b1 - 1; u >= b0; u--) {
+      if (is_leaf(u) || !active_[u]) continue;
+      emit_reverse(u);
+    }
+    for (auto& io : ins) partial_of_[io.first] = -1;
+    for (int u = b0; u < b1; u++) body_adj_[u] = -1;
+    cur_region_ = -1;
+    block_vr_ = -1;
+  }
+  mult_ = 1.0;
+  PInst el; el.d.op = D_ENDLOOP; el.f[0] = I(loop_pc);
+  int end_pc = emit(el);
+  code_[loop_pc].f[3] = I(end_pc);
+  PInst gr; gr.d.op = D_GREDUCE; gr.f[0] = R(slotref(block)); gr.f[1] = I(1 + (int)ins.size());
+  emit(gr);
+}
+
+int32_t Planner::encode(const PArg& a) const {
+  if (!a.isref) return a.v;
+  if (a.r.kind == RK_SLOT) {
+    const VR& vr = vrs_[a.r.id];
+    if (vr.phys < 0) unsupported("internal: unallocated slot");
+    return mkref(RK_SLOT, vr.phys + a.r.off);
+  }
+  return mkref(a.r.kind, a.r.id + a.r.off);
+}
+
+// Liveness over the linear instruction stream and first-fit allocation of
+// contiguous slot ranges (closed intervals: an output never aliases an input).
+void Planner::allocate() {
+  auto touch = [&](const PArg& a, int pos) {
+    if (!a.isref || a.r.kind != RK_SLOT) return;
+    VR& vr = vrs_[a.r.id];
+    vr.start = std::min(vr.start, pos);
+    vr.end = std::max(vr.end, pos);
+  };
+  for (int pc = 0; pc < (int)code_.size(); pc++) {
+    const PInst& p = code_[pc];
+    for (int k = 0; k < 8; k++) touch(p.f[k], pc);
+    int off = -1, cnt = 0, stride = 1;
+    switch (p.d.op) {
+      case D_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 1; break;
+      case B_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 2; break;
+      case B_DSUM: off = p.f[1].v; cnt = p.f[2].v; stride = 3; break;
+      default: break;
+    }
+    if (off >= 0)
+      for (int e = 0; e < cnt * stride; e++) touch(args_[off + e], pc);
+  }
+  // values live across a data-axis loop stay live to its end
+  for (int pc = 0; pc < (int)code_.size(); pc++) {
+    if (code_[pc].d.op != D_LOOP) continue;
+    int end = code_[pc].f[3].v;
+    for (VR& vr : vrs_)
+      if (vr.start < pc && vr.end >= pc && vr.end < end) vr.end = end;
+  }
+  std::vector<int> order;
+  for (int i = 0; i < (int)vrs_.size(); i++) if (vrs_[i].end >= 0) order.push_back(i);
+  std::sort(order.begin(), order.end(), [&](int a, int b) {
+    if (vrs_[a].start != vrs_[b].start) return vrs_[a].start < vrs_[b].start;
+    return a < b;
+  });
+  std::vector<int> busy_until;  // per physical slot: last position it is occupied
+  for (int id : order) {
+    VR& vr = vrs_[id];
+    int w = vr.width, run = 0, base = -1;
+    for (int s = 0; s < (int)busy_until.size(); s++) {
+      if (busy_until[s] < vr.start) { if (++run == w) { base = s - w + 1; break; } }
+      else run = 0;
+    }
+    if (base < 0) {
+      base = (int)busy_until.size() - run;
+      busy_until.resize(base + w, -1);
+    }
+    for (int s = base; s < base + w; s++) busy_until[s] = vr.end;
+    vr.phys = base;
+  }
+  n_slots_ = (int)busy_until.size();
+}
+
+Plan Planner::build() {
+  // a shared constant 1.0 for seeds of lane-level region results
+  one_const_ = -1;
+  for (size_t k = 0; k < T.consts.size(); k++) {
+    double one = 1.0;
+    if (std::memcmp(&T.consts[k], &one, 8) == 0) { one_const_ = (int)k; break; }
+  }
+  if (one_const_ < 0) { extra_consts_.push_back(1.0); one_const_ = (int)T.consts.size(); }
+  if (T.loss < 0 || T.loss >= (int)T.nodes.size()) unsupported("tape has no loss");
+  analyze();
+  Plan pl;
+  pl.grad = grad_;
+  pl.spill = spill_;
+  // forward sweep
+  for (int v = 0; v < N; v++) {
+    if (is_leaf(v) || region_body_[v]) continue;
+    if (T.nodes[v].op == OP_DSUM) { pl.has_regions = true; emit_region(v); continue; }
+    emit_forward(v);
+  }
+  PInst ls; ls.d.op = D_LOSS; ls.f[0] = R(ref(T.loss));
+  emit(ls);
+  if (grad_) {
+    if (active_[T.loss]) {
+      if (is_leaf(T.loss)) {
+        adj_vr_[T.loss] = new_vr(1);
+      } else {
+        adj_vr_[T.loss] = new_vr(1);
+      }
+      PInst sd; sd.d.op = D_SEED; sd.f[0] = R(slotref(adj_vr_[T.loss]));
+      emit(sd);
+      for (int v = N - 1; v >= 0; v--) {
+        if (is_leaf(v) || region_body_[v] || !active_[v]) continue;
+        emit_reverse(v);
+      }
+    }
+    // parameter gradients: a PARAM leaf's adjoint is the gradient
+    std::vector<int> pnode(T.n_params, -1);
+    for (int v = 0; v < N; v++) if (T.nodes[v].op == OP_PARAM) pnode[T.nodes[v].imm] = v;
+    for (int k = 0; k < T.n_params; k++) {
+      PInst g; g.d.op = B_GRAD;
+      int v = pnode[k];
+      if (v >= 0 && adj_vr_[v] >= 0) g.f[0] = R(slotref(adj_vr_[v]));
+      g.f[1] = I(k);
+      emit(g);
+    }
+  }
+  allocate();
+  pl.n_slots = n_slots_;
+  pl.n_save = S_;
+  pl.n_params = T.n_params;
+  pl.n_obs_min = T.n_obs_min;
+  for (const Node& nd : T.nodes) if (nd.op == OP_DOBS && nd.imm > pl.max_dobs) pl.max_dobs = nd.imm;
+  for (const PInst& p : code_) {
+    DInst d = p.d;
+    for (int k = 0; k < 8; k++) d.f[k] = encode(p.f[k]);
+    pl.code.push_back(d);
+  }
+  for (const PArg& a : args_) pl.args.push_back(encode(a));
+  pl.extra_consts = extra_consts_;
+  pl.work_fwd = work_fwd_;
+  pl.work_rev = work_rev_;
+  pl.n_ops_per_lane = nops_;
+  return pl;
+}
+
+}  // namespace
+
+Plan make_plan(const Tape& t, bool grad, int force_mode) {
+  if (force_mode == 0 || force_mode == 1) return Planner(t, grad, force_mode == 1).build();
+  Plan keep = Planner(t, grad, false).build();
+  if (!grad || keep.n_slots <= 192) return keep;
+  return Planner(t, grad, true).build();
+}
+
+bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
+  const size_t nconst = n_consts + p.extra_consts.size();
+  // ref: any readable operand; slot: a writable slot reference
+  auto ref_ok = [&](int32_t r, int64_t width, bool must_slot) -> bool {
+    if (r == -1) return true;
+    if (width < 1) width = 1;
+    uint32_t kind = ref_kind(r);
+    int64_t idx = ref_index(r);
+    if (must_slot && kind != RK_SLOT) return false;
+    switch (kind) {
+      case RK_SLOT: return idx + width <= p.n_slots;
+      case RK_CONST: return (size_t)(idx + width) <= nconst;
+      case RK_OBS: return idx + width <= p.n_obs_min;
+      case RK_DOBS: return idx + width - 1 <= p.max_dobs;
+      case RK_SAVE: return idx + width <= p.n_save;
+      case RK_PARAM: return idx + width <= p.n_params;
+      default: return false;
+    }
+  };
+  auto save_ok = [&](int32_t s, int64_t width) { return s == -1 || (s >= 0 && s + width <= p.n_save); };
+  auto args_ok = [&](int32_t off, int64_t cnt, int stride) {
+    return off >= 0 && cnt >= 0 && (size_t)off + (size_t)cnt * stride <= p.args.size();
+  };
+  int open_loop = -1;
+  for (size_t pc = 0; pc < p.code.size(); pc++) {
+    const DInst& d = p.code[pc];
+    const int32_t* f = d.f;
+    const int r = d.r, c = d.c, k = d.k, w = r * c, n = d.r;
+    bool ok = true;
+    if (r < 1 || c < 1 || r > 16 || c > 16 || ((d.op == D_MATMUL || d.op == B_MATMUL) && (k < 1 || k > 16)) ||
+        (d.op == D_CMP && k > 4)) {
+      why = "bad shape";
+      return false;
+    }
+    switch (d.op) {
+      case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: case D_CMP:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && ref_ok(f[2], 1, false) && save_ok(f[3], 1);
+        break;
+      case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: case D_POWI:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && save_ok(f[3], 1) && (d.op != D_POWI || (f[7] >= 0 && f[7] <= 64));
+        break;
+      case D_SIN: case D_COS:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && save_ok(f[3], 1) && ref_ok(f[4], 1, true) && save_ok(f[5], 1);
+        break;
+      case D_SELECT:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && ref_ok(f[2], 1, false) && ref_ok(f[4], 1, false) && save_ok(f[3], 1);
+        break;
+      case D_GATHER:
+        ok = ref_ok(f[0], f[2], true) && args_ok(f[1], f[2], 1) && save_ok(f[3], f[2]);
+        if (ok) for (int e = 0; e < f[2]; e++) ok = ok && ref_ok(p.args[f[1] + e], 1, false);
+        break;
+      case D_MADD: case D_MSUB:
+        ok = ref_ok(f[0], w, true) && ref_ok(f[1], w, false) && ref_ok(f[2], w, false) && save_ok(f[3], w);
+        break;
+      case D_MSCALE:
+        ok = ref_ok(f[0], w, true) && ref_ok(f[1], 1, false) && ref_ok(f[2], w, false) && save_ok(f[3], w);
+        break;
+      case D_MATMUL:
+        ok = ref_ok(f[0], w, true) && ref_ok(f[1], r * k, false) && ref_ok(f[2], k * c, false) && save_ok(f[3], w);
+        break;
+      case D_INV:
+        ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, false) && save_ok(f[3], n * n);
+        break;
+      case D_DET: case D_LOGDET:
+        ok = n <= 8 && ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, false) && save_ok(f[3], 1) &&
+             ref_ok(f[4], n * n, true) && save_ok(f[5], n * n);
+        break;
+      case D_TRACE: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, false); break;
+      case D_ZERO: case D_GREDUCE: ok = f[1] >= 0 && ref_ok(f[0], f[1], true); break;
+      case D_LOOP:
+        ok = open_loop < 0 && f[3] > (int)pc && f[3] < (int)p.code.size() && p.code[f[3]].op == D_ENDLOOP &&
+             f[0] >= 0 && f[1] >= 0 && f[2] >= 0;
+        open_loop = (int)pc;
+        break;
+      case D_ENDLOOP: ok = f[0] == open_loop && p.code[f[0]].f[3] == (int)pc; open_loop = -1; break;
+      case D_ACC: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false); break;
+      case D_SEED: ok = ref_ok(f[0], 1, true); break;
+      case D_LOSS: ok = ref_ok(f[0], 1, false); break;
+      case B_ADD: case B_SUB: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true); break;
+      case B_NEG: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true); break;
+      case B_MUL: case B_DIV: case B_POW:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true) && ref_ok(f[3], 1, false) &&
+             ref_ok(f[4], 1, false) && ref_ok(f[5], 1, false);
+        break;
+      case B_EXP: case B_TANH: case B_LOG: case B_ABS: case B_SQRT: case B_SIN: case B_COS: case B_POWI:
+        ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[3], 1, false) && ref_ok(f[5], 1, false) &&
+             ref_ok(f[6], 1, false) && (d.op != B_POWI || (f[7] >= 0 && f[7] <= 64));
+        break;
+      case B_SELECT: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true) && ref_ok(f[3], 1, false); break;
+      case B_GATHER:
+        ok = ref_ok(f[0], f[2], true) && args_ok(f[1], f[2], 2);
+        if (ok) for (int e = 0; e < f[2]; e++) ok = ok && ref_ok(p.args[f[1] + 2 * e], 1, true);
+        break;
+      case B_SCATTER:
+        ok = ref_ok(f[0], f[2], true) && ref_ok(f[1], f[4], true) && args_ok(f[3], f[2], 1) && f[4] >= 1 && f[4] <= 256;
+        if (ok) for (int e = 0; e < f[2]; e++) ok = ok && p.args[f[3] + e] >= 0 && p.args[f[3] + e] < f[4];
+        break;
+      case B_MADD: case B_MSUB: ok = ref_ok(f[0], w, true) && ref_ok(f[1], w, true) && ref_ok(f[2], w, true); break;
+      case B_MSCALE:
+        ok = ref_ok(f[0], w, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], w, true) && ref_ok(f[3], 1, false) && ref_ok(f[4], w, false);
+        break;
+      case B_MATMUL:
+        ok = ref_ok(f[0], w, true) && ref_ok(f[1], r * k, true) && ref_ok(f[2], k * c, true) && ref_ok(f[3], r * k, false) &&
+             ref_ok(f[4], k * c, false);
+        break;
+      case B_INV: ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, true) && ref_ok(f[5], n * n, false); break;
+      case B_DET: case B_LOGDET:
+        ok = n <= 8 && ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, true) && ref_ok(f[5], 1, false) && ref_ok(f[6], n * n, false);
+        break;
+      case B_TRACE: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, true); break;
+      case B_DSUM:
+        ok = ref_ok(f[0], 1, true) && args_ok(f[1], f[2], 3);
+        if (ok)
+          for (int e = 0; e < f[2]; e++)
+            ok = ok && ref_ok(p.args[f[1] + 3 * e], 1, true) && p.args[f[1] + 3 * e] != -1 && ref_ok(p.args[f[1] + 3 * e + 2], 1, true);
+        break;
+      case B_GRAD: ok = ref_ok(f[0], 1, true) && f[1] >= 0 && f[1] < p.n_params; break;
+      default: why = "bad opcode"; return false;
+    }
+    if (!ok) { why = "operand out of range at instruction " + std::to_string(pc) + " (op " + std::to_string(d.op) + ")"; return false; }
+  }
+  if (open_loop >= 0) { why = "unterminated loop"; return false; }
+  return true;
+}
+
+}  // namespace ndvm

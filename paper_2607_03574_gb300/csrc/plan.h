@@ -1,0 +1,107 @@
+// Device program ("plan") for tape replay, produced on the host from a Tape.
+//
+// The kernel interprets a linear instruction stream.  Every lane runs the same
+// stream (the tape is shared by the population, section 3.5), so dispatch is
+// uniform across a warp.  Per-lane values live in a slot file in shared memory,
+// laid out [slot][thread]; the planner register-allocates slots by liveness.
+// Values that the reverse sweep reads are either kept in slots until then (short
+// tapes) or stored to an HBM workspace laid out [element][lane] (lane-contiguous,
+// coalesced) and read back in the reverse sweep (long tapes).
+#pragma once
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "tape.h"
+
+namespace ndvm {
+
+// Operand reference: kind in bits 28..30, index in bits 0..27; element e of a
+// matrix operand is ref + e.  -1 means "none".
+enum RefKind : uint32_t { RK_SLOT = 0, RK_CONST = 1, RK_OBS = 2, RK_DOBS = 3, RK_SAVE = 4, RK_PARAM = 5 };
+constexpr int32_t kRefIndexMask = 0x0fffffff;
+inline int32_t mkref(uint32_t kind, int32_t idx) { return (int32_t)((kind << 28) | (uint32_t)idx); }
+inline uint32_t ref_kind(int32_t r) { return ((uint32_t)r >> 28) & 7u; }
+inline int32_t ref_index(int32_t r) { return r & kRefIndexMask; }
+
+enum DOp : uint8_t {
+  // ---- forward ----
+  D_ADD = 1, D_SUB, D_MUL, D_DIV, D_POW,  // f0 out, f1 a, f2 b, f3 save
+  D_NEG, D_EXP, D_LOG, D_TANH, D_SQRT, D_ABS,  // f0 out, f1 a, f3 save
+  D_SIN, D_COS,     // f0 out, f1 a, f3 save, f4 aux slot (the other trig value), f5 aux save
+  D_POWI,           // f0 out, f1 a, f3 save, f7 n
+  D_CMP,            // f0 out, f1 a, f2 b, k = comparison (0 lt, 1 le, 2 gt, 3 ge, 4 eq)
+  D_SELECT,         // f0 out, f1 predicate, f2 a, f3 save, f4 b
+  D_GATHER,         // f0 out, f1 args offset, f2 count (args: element refs), f3 save
+  D_MADD, D_MSUB,   // f0 out, f1 a, f2 b, f3 save; r x c
+  D_MSCALE,         // f0 out, f1 s, f2 A, f3 save; r x c
+  D_MATMUL,         // f0 out, f1 A, f2 B, f3 save; r x c, inner k
+  D_INV,            // f0 out, f1 A, f3 save; n = r
+  D_DET, D_LOGDET,  // f0 out, f1 A, f3 save, f4 aux slot (inverse), f5 aux save; n = r
+  D_TRACE,          // f0 out, f1 A; n = r
+  // ---- data-axis regions ----
+  D_ZERO,           // f0 slot, f1 count
+  D_LOOP,           // f0 N, f1 stride, f2 base, f3 pc of the matching D_ENDLOOP
+  D_ENDLOOP,        // f0 pc of the matching D_LOOP
+  D_ACC,            // slot f0 += ref f1
+  D_SEED,           // slot f0 = 1
+  D_GREDUCE,        // f0 slot, f1 count: sum over the lane's thread group
+  D_LOSS,           // loss[lane] = ref f0
+  // ---- reverse ----  (f0 = adjoint of the output "gz"; targets f1/f2; flags bit0/bit1 = first
+  //                     contribution to target 1/2, which stores instead of accumulating)
+  B_ADD, B_SUB,     // f1 ga, f2 gb
+  B_MUL,            // f1 ga, f2 gb, f3 pa, f4 pb
+  B_DIV,            // f1 ga, f2 gb, f4 pb, f5 pz
+  B_POW,            // f1 ga, f2 gb, f3 pa, f4 pb, f5 pz
+  B_NEG,            // f1 ga
+  B_EXP, B_TANH,    // f1 ga, f5 pz
+  B_LOG, B_ABS,     // f1 ga, f3 pa
+  B_SQRT,           // f1 ga, f3 pa, f5 pz
+  B_SIN, B_COS,     // f1 ga, f6 paux (cos x for sin, sin x for cos)
+  B_POWI,           // f1 ga, f3 pa, f7 n
+  B_SELECT,         // f1 ga, f2 gb, f3 pp
+  B_GATHER,         // f1 args offset, f2 count (args: pairs target slot|-1, first flag)
+  B_SCATTER,        // f1 ga, f2 count, f3 args offset (input element per output), f4 input width
+  B_MADD, B_MSUB,   // f1 ga, f2 gb; r x c
+  B_MSCALE,         // f1 gs, f2 gA, f3 ps, f4 pA; r x c
+  B_MATMUL,         // f1 gA, f2 gB, f3 pA, f4 pB; r x c, inner k
+  B_INV,            // f1 gA, f5 pz; n = r
+  B_DET,            // f1 gA, f5 pz, f6 pinv; n = r
+  B_LOGDET,         // f1 gA, f6 pinv; n = r
+  B_TRACE,          // f1 gA; n = r
+  B_DSUM,           // f1 args offset, f2 count (args: triples target slot, first flag, partial slot)
+  B_GRAD,           // grad[lane, f1] = slot f0 (or 0 if f0 < 0)
+  D_NOPS
+};
+
+struct DInst {
+  uint8_t op = 0, r = 1, c = 1, k = 1;
+  uint8_t flags = 0, pad0 = 0, pad1 = 0, pad2 = 0;
+  int32_t f[8] = {-1, -1, -1, -1, -1, -1, -1, -1};
+};
+static_assert(sizeof(DInst) == 40, "DInst layout");
+
+struct Plan {
+  bool grad = false;          // has a reverse sweep
+  bool spill = false;         // reverse reads primals from the HBM workspace
+  bool has_regions = false;   // contains data-axis loops
+  int32_t n_slots = 0;        // per-lane slot file size (elements)
+  int64_t n_save = 0;         // per-lane workspace elements
+  int32_t n_params = 0;
+  int64_t n_obs_min = 0;
+  int32_t max_dobs = -1;      // largest DOBS column read (for validation)
+  std::vector<DInst> code;
+  std::vector<int32_t> args;
+  std::vector<double> extra_consts;  // appended after the tape's constant pool
+  // algorithmic cost per lane (for the roofline): DFMA-equivalents and saved bytes
+  double work_fwd = 0, work_rev = 0;
+  double n_ops_per_lane = 0;
+};
+
+// Build the plan; throws BuildError on unsupported tapes.
+Plan make_plan(const Tape& t, bool grad, int force_mode = -1 /* -1 auto, 0 keep, 1 spill */);
+
+// Check every reference against the plan's own sizes (host-side, before upload).
+bool validate_plan(const Plan& p, size_t n_consts, std::string& why);
+
+}  // namespace ndvm

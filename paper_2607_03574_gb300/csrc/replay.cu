@@ -1,0 +1,648 @@
+// Tape replay on the GPU (sm_103a): forward sweep, reverse adjoint sweep and
+// per-lane loss for a population of parameter lanes (paper sections 3.4-3.5,
+// Appendix C).
+//
+// Execution model.  Every lane runs the same instruction stream (the tape is
+// shared by the population), so instruction fetch and dispatch are uniform across
+// a warp; the stream is read through the read-only data path and broadcast.  A
+// group of G consecutive threads serves one lane (G = 1 except for tapes with
+// data-axis regions, where the group splits the lane's data points and reduces
+// partial sums with warp shuffles).  Each thread owns a slot file of R values in
+// shared memory, laid out [slot][thread] so a warp touches 32 consecutive
+// elements per slot.  Forward values read by the reverse sweep are either kept in
+// slots (short tapes) or stored to the workspace as [element][lane] -- each warp
+// store/load is one contiguous, coalesced run -- and read back in reverse.
+//
+// GB300 note: FP64 issues at about 1/73 of the FP32 rate, so the interpreter's
+// integer dispatch, shared-memory traffic and branches hide under the FP64 pipe;
+// the cost of a replay is the FP64 work it issues.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "plan.h"
+#include "replay.h"
+
+namespace ndvm {
+namespace {
+
+template <typename T>
+struct Opnd {
+  const T* p;
+  int64_t s;
+  __device__ __forceinline__ T operator[](int e) const { return p[(int64_t)e * s]; }
+};
+
+template <typename T>
+struct Lane {
+  T* slots;
+  int tpb, tid;
+  const T* consts;
+  const T* obs;
+  const T* params;
+  T* save;
+  int64_t lane, col, save_ld, dbase;
+  int P;
+
+  __device__ __forceinline__ Opnd<T> rd(int32_t ref) const {
+    const uint32_t kind = ((uint32_t)ref >> 28) & 7u;
+    const int32_t idx = ref & kRefIndexMask;
+    switch (kind) {
+      case RK_SLOT: return {slots + (int64_t)idx * tpb + tid, tpb};
+      case RK_CONST: return {consts + idx, 1};
+      case RK_OBS: return {obs + idx, 1};
+      case RK_DOBS: return {obs + dbase + idx, 1};
+      case RK_SAVE: return {save + (int64_t)idx * save_ld + col, save_ld};
+      default: return {params + lane * P + idx, 1};
+    }
+  }
+  __device__ __forceinline__ T ld(int32_t ref) const { return rd(ref)[0]; }
+  // slot references only
+  __device__ __forceinline__ T* wp(int32_t ref) const { return slots + (int64_t)(ref & kRefIndexMask) * tpb + tid; }
+  __device__ __forceinline__ void st(int32_t ref, int e, T v) const { wp(ref)[(int64_t)e * tpb] = v; }
+  __device__ __forceinline__ T sl(int32_t ref, int e) const { return wp(ref)[(int64_t)e * tpb]; }
+  // adjoint update: first contribution stores, later ones accumulate
+  __device__ __forceinline__ void upd(int32_t ref, int e, T v, bool first) const {
+    T* q = wp(ref) + (int64_t)e * tpb;
+    *q = first ? v : *q + v;
+  }
+  __device__ __forceinline__ void save_out(int32_t sidx, int e, T v) const {
+    if (sidx >= 0) save[(int64_t)(sidx + e) * save_ld + col] = v;
+  }
+};
+
+template <typename T> __device__ __forceinline__ T clamp_eps() { return (T)1e-8; }
+
+template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
+  if (n == 0) return (T)1;
+  T z = a;
+  for (int i = 1; i < n; i++) z = z * a;
+  return z;
+}
+
+// determinant and (optionally) inverse of an n x n matrix read from an operand
+// (closed-form adjugate for n <= 3, Gauss-Jordan with partial pivoting above)
+template <typename T>
+__device__ T det_inv(const Opnd<T>& A, int n, T* inv /* n*n or nullptr */) {
+  if (n == 1) {
+    T d = A[0];
+    if (inv) inv[0] = (T)1 / d;
+    return d;
+  }
+  if (n == 2) {
+    T a0 = A[0], a1 = A[1], a2 = A[2], a3 = A[3];
+    T d = a0 * a3 - a1 * a2;
+    if (inv) {
+      T r = (T)1 / d;
+      inv[0] = a3 * r; inv[1] = -a1 * r; inv[2] = -a2 * r; inv[3] = a0 * r;
+    }
+    return d;
+  }
+  if (n == 3) {
+    T a[9];
+#pragma unroll
+    for (int i = 0; i < 9; i++) a[i] = A[i];
+    T c00 = a[4] * a[8] - a[5] * a[7];
+    T c01 = a[5] * a[6] - a[3] * a[8];
+    T c02 = a[3] * a[7] - a[4] * a[6];
+    T d = a[0] * c00 + a[1] * c01 + a[2] * c02;
+    if (inv) {
+      T c10 = a[2] * a[7] - a[1] * a[8];
+      T c11 = a[0] * a[8] - a[2] * a[6];
+      T c12 = a[1] * a[6] - a[0] * a[7];
+      T c20 = a[1] * a[5] - a[2] * a[4];
+      T c21 = a[2] * a[3] - a[0] * a[5];
+      T c22 = a[0] * a[4] - a[1] * a[3];
+      T r = (T)1 / d;
+      inv[0] = c00 * r; inv[1] = c10 * r; inv[2] = c20 * r;
+      inv[3] = c01 * r; inv[4] = c11 * r; inv[5] = c21 * r;
+      inv[6] = c02 * r; inv[7] = c12 * r; inv[8] = c22 * r;
+    }
+    return d;
+  }
+  // n = 4..8: elimination on [A | I] in thread-local memory
+  T w[8][16];
+  for (int i = 0; i < n; i++)
+    for (int j = 0; j < 2 * n; j++) w[i][j] = j < n ? A[i * n + j] : (T)(j - n == i ? 1 : 0);
+  T d = (T)1;
+  for (int col = 0; col < n; col++) {
+    int piv = col;
+    T best = fabs(w[col][col]);
+    for (int i = col + 1; i < n; i++)
+      if (fabs(w[i][col]) > best) { best = fabs(w[i][col]); piv = i; }
+    if (piv != col) {
+      for (int j = 0; j < 2 * n; j++) { T t = w[col][j]; w[col][j] = w[piv][j]; w[piv][j] = t; }
+      d = -d;
+    }
+    T pv = w[col][col];
+    d = d * pv;
+    T r = (T)1 / pv;
+    for (int j = 0; j < 2 * n; j++) w[col][j] = w[col][j] * r;
+    for (int i = 0; i < n; i++) {
+      if (i == col) continue;
+      T f = w[i][col];
+      if (f != (T)0)
+        for (int j = 0; j < 2 * n; j++) w[i][j] = w[i][j] - f * w[col][j];
+    }
+  }
+  if (inv)
+    for (int i = 0; i < n; i++)
+      for (int j = 0; j < n; j++) inv[i * n + j] = w[i][n + j];
+  return d;
+}
+
+template <typename T>
+__device__ __forceinline__ bool all_zero(const Lane<T>& L, int32_t gz, int w) {
+  for (int e = 0; e < w; e++)
+    if (L.sl(gz, e) != (T)0) return false;
+  return true;
+}
+template <typename T>
+__device__ __forceinline__ void zero_if_first(const Lane<T>& L, int32_t ref, int w, bool first) {
+  if (first && ref != -1)
+    for (int e = 0; e < w; e++) L.st(ref, e, (T)0);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int tid = threadIdx.x;
+  const int tpb = blockDim.x;
+  const int G = 1 << a.log2g;
+  const int64_t lane_raw = a.lane0 + (int64_t)blockIdx.x * (tpb >> a.log2g) + (tid >> a.log2g);
+  const int grank = tid & (G - 1);
+  const bool live = lane_raw < a.lane_end;
+  if (G == 1 && !live) return;
+
+  Lane<T> L;
+  L.slots = reinterpret_cast<T*>(smem_raw);
+  L.tpb = tpb;
+  L.tid = tid;
+  L.consts = static_cast<const T*>(a.consts);
+  L.obs = static_cast<const T*>(a.obs);
+  L.params = static_cast<const T*>(a.params);
+  L.save = static_cast<T*>(a.save);
+  L.lane = live ? lane_raw : a.lane_end - 1;
+  L.col = L.lane - a.lane0;
+  L.save_ld = a.save_ld;
+  L.P = a.P;
+  L.dbase = 0;
+  T* loss = static_cast<T*>(a.loss);
+  T* grad = static_cast<T*>(a.grad);
+  const bool writer = live && grank == 0;
+
+  int64_t d = 0, dN = 0, dstride = 0, dbase0 = 0;
+  int loop_pc = -1;
+  const DInst* __restrict__ code = a.code;
+  const int32_t* __restrict__ args = a.args;
+
+  for (int pc = 0; pc < a.n_code; pc++) {
+    const DInst in = code[pc];
+    const int32_t* f = in.f;
+    const int w = in.r * in.c;
+    switch (in.op) {
+      // ------------------------------------------------------------ forward
+      case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: {
+        T x = L.ld(f[1]), y = L.ld(f[2]), z;
+        if (in.op == D_ADD) z = x + y;
+        else if (in.op == D_SUB) z = x - y;
+        else if (in.op == D_MUL) z = x * y;
+        else if (in.op == D_DIV) z = x / y;
+        else z = pow(x, y);
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: {
+        T x = L.ld(f[1]), z;
+        if (in.op == D_NEG) z = -x;
+        else if (in.op == D_EXP) z = exp(x);
+        else if (in.op == D_LOG) z = log(x > clamp_eps<T>() ? x : clamp_eps<T>());
+        else if (in.op == D_TANH) z = tanh(x);
+        else if (in.op == D_SQRT) z = sqrt(x > clamp_eps<T>() ? x : clamp_eps<T>());
+        else z = fabs(x);
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_SIN: case D_COS: {
+        T x = L.ld(f[1]);
+        T s, c;
+        if (f[4] != -1 || f[5] >= 0) {
+          sincos(x, &s, &c);
+          T aux = in.op == D_SIN ? c : s;
+          if (f[4] != -1) L.st(f[4], 0, aux);
+          L.save_out(f[5], 0, aux);
+        } else if (in.op == D_SIN) {
+          s = sin(x);
+        } else {
+          c = cos(x);
+        }
+        T z = in.op == D_SIN ? s : c;
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_POWI: {
+        T z = powi_rep(L.ld(f[1]), f[7]);
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_CMP: {
+        T x = L.ld(f[1]), y = L.ld(f[2]);
+        bool r = in.k == 0 ? x < y : in.k == 1 ? x <= y : in.k == 2 ? x > y : in.k == 3 ? x >= y : x == y;
+        T z = r ? (T)1 : (T)0;
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_SELECT: {
+        T p = L.ld(f[1]);
+        T z = p != (T)0 ? L.ld(f[2]) : L.ld(f[4]);
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
+      case D_GATHER: {
+        const int32_t* g = args + f[1];
+        for (int e = 0; e < f[2]; e++) {
+          T v = L.ld(g[e]);
+          L.st(f[0], e, v);
+          L.save_out(f[3], e, v);
+        }
+        break;
+      }
+      case D_MADD: case D_MSUB: {
+        Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
+        for (int e = 0; e < w; e++) {
+          T z = in.op == D_MADD ? A[e] + Bm[e] : A[e] - Bm[e];
+          L.st(f[0], e, z);
+          L.save_out(f[3], e, z);
+        }
+        break;
+      }
+      case D_MSCALE: {
+        T s = L.ld(f[1]);
+        Opnd<T> A = L.rd(f[2]);
+        for (int e = 0; e < w; e++) {
+          T z = s * A[e];
+          L.st(f[0], e, z);
+          L.save_out(f[3], e, z);
+        }
+        break;
+      }
+      case D_MATMUL: {
+        Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
+        const int r = in.r, c = in.c, kk = in.k;
+        for (int i = 0; i < r; i++)
+          for (int j = 0; j < c; j++) {
+            T s = A[i * kk] * Bm[j];
+            for (int q = 1; q < kk; q++) s = fma(A[i * kk + q], Bm[q * c + j], s);
+            L.st(f[0], i * c + j, s);
+            L.save_out(f[3], i * c + j, s);
+          }
+        break;
+      }
+      case D_INV: {
+        const int n = in.r;
+        T inv[64];
+        det_inv(L.rd(f[1]), n, inv);
+        for (int e = 0; e < n * n; e++) {
+          L.st(f[0], e, inv[e]);
+          L.save_out(f[3], e, inv[e]);
+        }
+        break;
+      }
+      case D_DET: case D_LOGDET: {
+        const int n = in.r;
+        const bool aux = f[4] != -1 || f[5] >= 0;
+        T inv[64];
+        T dt = det_inv(L.rd(f[1]), n, aux ? inv : nullptr);
+        T z = in.op == D_DET ? dt : log(dt);
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        if (aux)
+          for (int e = 0; e < n * n; e++) {
+            if (f[4] != -1) L.st(f[4], e, inv[e]);
+            L.save_out(f[5], e, inv[e]);
+          }
+        break;
+      }
+      case D_TRACE: {
+        const int n = in.r;
+        Opnd<T> A = L.rd(f[1]);
+        T s = A[0];
+        for (int i = 1; i < n; i++) s = s + A[i * n + i];
+        L.st(f[0], 0, s);
+        break;
+      }
+      // ------------------------------------------------------------ data axis
+      case D_ZERO:
+        for (int e = 0; e < f[1]; e++) L.st(f[0], e, (T)0);
+        break;
+      case D_LOOP:
+        dN = f[0]; dstride = f[1]; dbase0 = f[2];
+        d = grank;
+        loop_pc = pc;
+        if (d >= dN) { pc = f[3]; break; }  // resumes after the loop end
+        L.dbase = dbase0 + d * dstride;
+        break;
+      case D_ENDLOOP:
+        d += G;
+        if (d < dN) { L.dbase = dbase0 + d * dstride; pc = loop_pc; }
+        break;
+      case D_ACC: L.st(f[0], 0, L.sl(f[0], 0) + L.ld(f[1])); break;
+      case D_SEED: L.st(f[0], 0, (T)1); break;
+      case D_GREDUCE:
+        if (G > 1) {
+          __syncwarp();
+          for (int e = 0; e < f[1]; e++) {
+            T v = L.sl(f[0], e);
+            for (int o = G >> 1; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            L.st(f[0], e, v);
+          }
+        }
+        break;
+      case D_LOSS:
+        if (writer) loss[L.lane] = L.ld(f[0]);
+        break;
+      // ------------------------------------------------------------ reverse
+      case B_ADD: case B_SUB: case B_NEG: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); if (in.op != B_NEG) zero_if_first(L, f[2], 1, fb); break; }
+        if (f[1] != -1) L.upd(f[1], 0, in.op == B_NEG ? -g : g, fa);
+        if (in.op != B_NEG && f[2] != -1) L.upd(f[2], 0, in.op == B_ADD ? g : -g, fb);
+        break;
+      }
+      case B_MUL: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        if (f[1] != -1) L.upd(f[1], 0, g * L.ld(f[4]), fa);
+        if (f[2] != -1) L.upd(f[2], 0, g * L.ld(f[3]), fb);
+        break;
+      }
+      case B_DIV: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        T q = g / L.ld(f[4]);
+        if (f[1] != -1) L.upd(f[1], 0, q, fa);
+        if (f[2] != -1) L.upd(f[2], 0, -(q * L.ld(f[5])), fb);
+        break;
+      }
+      case B_POW: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        T x = L.ld(f[3]), e = L.ld(f[4]), z = L.ld(f[5]);
+        if (f[1] != -1) L.upd(f[1], 0, g * e * z / x, fa);
+        if (f[2] != -1) L.upd(f[2], 0, g * z * log(x), fb);
+        break;
+      }
+      case B_EXP: case B_TANH: case B_LOG: case B_ABS: case B_SQRT: case B_SIN: case B_COS: case B_POWI: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1;
+        if (f[1] == -1) break;
+        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); break; }
+        T v;
+        switch (in.op) {
+          case B_EXP: v = g * L.ld(f[5]); break;
+          case B_TANH: { T z = L.ld(f[5]); v = g * ((T)1 - z * z); break; }
+          case B_LOG: { T x = L.ld(f[3]); v = x > clamp_eps<T>() ? g / x : (T)0; break; }
+          case B_ABS: { T x = L.ld(f[3]); v = x > (T)0 ? g : (x < (T)0 ? -g : g * (T)0); break; }
+          case B_SQRT: { T x = L.ld(f[3]); v = x > clamp_eps<T>() ? g / ((T)2 * L.ld(f[5])) : (T)0; break; }
+          case B_SIN: v = g * L.ld(f[6]); break;
+          case B_COS: v = -(g * L.ld(f[6])); break;
+          default: {  // POWI
+            int n = f[7];
+            v = n > 0 ? g * ((T)n * powi_rep(L.ld(f[3]), n - 1)) : (T)0;
+          }
+        }
+        L.upd(f[1], 0, v, fa);
+        break;
+      }
+      case B_SELECT: {
+        T g = L.sl(f[0], 0);
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        bool taken = L.ld(f[3]) != (T)0;
+        if (f[1] != -1) { if (taken && g != (T)0) L.upd(f[1], 0, g, fa); else zero_if_first(L, f[1], 1, fa); }
+        if (f[2] != -1) { if (!taken && g != (T)0) L.upd(f[2], 0, g, fb); else zero_if_first(L, f[2], 1, fb); }
+        break;
+      }
+      case B_GATHER: {
+        const int32_t* g = args + f[1];
+        const bool z = all_zero(L, f[0], f[2]);
+        for (int e = 0; e < f[2]; e++) {
+          int32_t t = g[2 * e];
+          if (t == -1) continue;
+          bool first = g[2 * e + 1] != 0;
+          if (z) zero_if_first(L, t, 1, first);
+          else L.upd(t, 0, L.sl(f[0], e), first);
+        }
+        break;
+      }
+      case B_SCATTER: {
+        if (f[1] == -1) break;
+        const bool first = in.flags & 1;
+        zero_if_first(L, f[1], f[4], first);
+        if (all_zero(L, f[0], f[2])) break;
+        const int32_t* m = args + f[3];
+        for (int e = 0; e < f[2]; e++) L.st(f[1], m[e], L.sl(f[1], m[e]) + L.sl(f[0], e));
+        break;
+      }
+      case B_MADD: case B_MSUB: {
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], w, fa); zero_if_first(L, f[2], w, fb); break; }
+        for (int e = 0; e < w; e++) {
+          T g = L.sl(f[0], e);
+          if (f[1] != -1) L.upd(f[1], e, g, fa);
+          if (f[2] != -1) L.upd(f[2], e, in.op == B_MADD ? g : -g, fb);
+        }
+        break;
+      }
+      case B_MSCALE: {
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], w, fb); break; }
+        if (f[1] != -1) {
+          Opnd<T> A = L.rd(f[4]);
+          T s = L.sl(f[0], 0) * A[0];
+          for (int e = 1; e < w; e++) s = fma(L.sl(f[0], e), A[e], s);
+          L.upd(f[1], 0, s, fa);
+        }
+        if (f[2] != -1) {
+          T s = L.ld(f[3]);
+          for (int e = 0; e < w; e++) L.upd(f[2], e, s * L.sl(f[0], e), fb);
+        }
+        break;
+      }
+      case B_MATMUL: {
+        const int r = in.r, c = in.c, kk = in.k;
+        bool fa = in.flags & 1, fb = in.flags & 2;
+        if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], r * kk, fa); zero_if_first(L, f[2], kk * c, fb); break; }
+        Opnd<T> G_ = {L.wp(f[0]), L.tpb};
+        if (f[1] != -1) {  // gA (r x k) += gZ (r x c) * B^T (B is k x c)
+          Opnd<T> Bm = L.rd(f[4]);
+          for (int i = 0; i < r; i++)
+            for (int q = 0; q < kk; q++) {
+              T s = G_[i * c] * Bm[q * c];
+              for (int j = 1; j < c; j++) s = fma(G_[i * c + j], Bm[q * c + j], s);
+              L.upd(f[1], i * kk + q, s, fa);
+            }
+        }
+        if (f[2] != -1) {  // gB (k x c) += A^T (A is r x k) * gZ
+          Opnd<T> A = L.rd(f[3]);
+          for (int q = 0; q < kk; q++)
+            for (int j = 0; j < c; j++) {
+              T s = A[q] * G_[j];
+              for (int i = 1; i < r; i++) s = fma(A[i * kk + q], G_[i * c + j], s);
+              L.upd(f[2], q * c + j, s, fb);
+            }
+        }
+        break;
+      }
+      case B_INV: {
+        const int n = in.r;
+        bool fa = in.flags & 1;
+        if (f[1] == -1) break;
+        if (all_zero(L, f[0], n * n)) { zero_if_first(L, f[1], n * n, fa); break; }
+        Opnd<T> Bv = L.rd(f[5]);
+        Opnd<T> G_ = {L.wp(f[0]), L.tpb};
+        T m[64];  // M = gZ B^T
+        for (int p = 0; p < n; p++)
+          for (int j = 0; j < n; j++) {
+            T s = G_[p * n] * Bv[j * n];
+            for (int q = 1; q < n; q++) s = fma(G_[p * n + q], Bv[j * n + q], s);
+            m[p * n + j] = s;
+          }
+        for (int i = 0; i < n; i++)  // gA -= B^T M
+          for (int j = 0; j < n; j++) {
+            T s = Bv[i] * m[j];
+            for (int p = 1; p < n; p++) s = fma(Bv[p * n + i], m[p * n + j], s);
+            L.upd(f[1], i * n + j, -s, fa);
+          }
+        break;
+      }
+      case B_DET: case B_LOGDET: {
+        const int n = in.r;
+        bool fa = in.flags & 1;
+        if (f[1] == -1) break;
+        T g = L.sl(f[0], 0);
+        if (g == (T)0) { zero_if_first(L, f[1], n * n, fa); break; }
+        T fac = in.op == B_DET ? g * L.ld(f[5]) : g;
+        Opnd<T> Iv = L.rd(f[6]);
+        for (int i = 0; i < n; i++)
+          for (int j = 0; j < n; j++) L.upd(f[1], i * n + j, fac * Iv[j * n + i], fa);
+        break;
+      }
+      case B_TRACE: {
+        const int n = in.r;
+        bool fa = in.flags & 1;
+        if (f[1] == -1) break;
+        T g = L.sl(f[0], 0);
+        zero_if_first(L, f[1], n * n, fa);
+        if (g == (T)0) break;
+        for (int i = 0; i < n; i++) L.st(f[1], i * n + i, L.sl(f[1], i * n + i) + g);
+        break;
+      }
+      case B_DSUM: {
+        T g = L.sl(f[0], 0);
+        const int32_t* q = args + f[1];
+        for (int e = 0; e < f[2]; e++) {
+          int32_t t = q[3 * e];
+          bool first = q[3 * e + 1] != 0;
+          if (g == (T)0) zero_if_first(L, t, 1, first);
+          else L.upd(t, 0, g * L.sl(q[3 * e + 2], 0), first);
+        }
+        break;
+      }
+      case B_GRAD:
+        if (writer) grad[L.lane * L.P + f[1]] = f[0] == -1 ? (T)0 : L.sl(f[0], 0);
+        break;
+      default:
+        if (a.err) atomicExch(a.err, 1);
+        return;
+    }
+  }
+}
+
+template <typename T>
+cudaError_t launch_t(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  static int configured_dev = -1;
+  static size_t configured_smem = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured_dev != dev || smem > configured_smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_replay<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured_dev = dev;
+    configured_smem = smem;
+  }
+  k_replay<T><<<blocks, tpb, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  return f32 ? launch_t<float>(a, blocks, tpb, smem, s) : launch_t<double>(a, blocks, tpb, smem, s);
+}
+
+}  // namespace ndvm
+
+// ---------------------------------------------------------------------------
+// FP64 peak probe: the roofline denominator of this FP64-bound path, measured on
+// the device in the same process as the replay.  Eight independent fused
+// multiply-add chains per thread, four 256-thread blocks per SM.
+namespace ndvm {
+namespace {
+__global__ void __launch_bounds__(256) k_dfma_peak(double* out, int iters) {
+  double a[8];
+  const double y = 0.999999999, c = 1e-9;
+#pragma unroll
+  for (int k = 0; k < 8; k++) a[k] = 1.0 + 1e-3 * k + 1e-7 * threadIdx.x;
+  for (int i = 0; i < iters; i++) {
+#pragma unroll
+    for (int k = 0; k < 8; k++) a[k] = fma(a[k], y, c);
+  }
+  double s = 0;
+#pragma unroll
+  for (int k = 0; k < 8; k++) s += a[k];
+  out[(size_t)blockIdx.x * blockDim.x + threadIdx.x] = s;
+}
+}  // namespace
+
+cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s) {
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int blocks = sms * 4, threads = 256, iters = 20000;
+  double* out = nullptr;
+  if ((e = cudaMalloc(&out, sizeof(double) * blocks * threads)) != cudaSuccess) return e;
+  cudaEvent_t e0, e1;
+  cudaEventCreate(&e0);
+  cudaEventCreate(&e1);
+  k_dfma_peak<<<blocks, threads, 0, s>>>(out, 200);  // warm-up
+  float best = 1e30f;
+  for (int rep = 0; rep < 3; rep++) {
+    cudaEventRecord(e0, s);
+    k_dfma_peak<<<blocks, threads, 0, s>>>(out, iters);
+    cudaEventRecord(e1, s);
+    e = cudaEventSynchronize(e1);
+    if (e != cudaSuccess) break;
+    float ms = 0;
+    cudaEventElapsedTime(&ms, e0, e1);
+    if (ms < best) best = ms;
+  }
+  if (e == cudaSuccess) e = cudaGetLastError();
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  cudaFree(out);
+  if (e == cudaSuccess) *flops_per_s = 2.0 * 8.0 * iters * (double)blocks * threads / (best * 1e-3);
+  return e;
+}
+}  // namespace ndvm

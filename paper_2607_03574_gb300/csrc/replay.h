@@ -1,0 +1,34 @@
+// Launch interface of the replay kernel (host side).
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "plan.h"
+
+namespace ndvm {
+
+struct ReplayArgs {
+  const DInst* code;     // device instruction stream
+  int n_code;
+  const int32_t* args;   // device operand lists
+  const void* consts;    // device constant pool in the compute type
+  const void* obs;       // device observations
+  const void* params;    // device B x P parameters
+  void* loss;            // device B losses
+  void* grad;            // device B x P gradients (gradient plans only)
+  void* save;            // device workspace [element][lane in chunk]
+  int64_t lane0;         // first lane of this launch
+  int64_t lane_end;      // one past the last lane of this launch
+  int64_t save_ld;       // workspace column count (lanes per chunk)
+  int P;
+  int log2g;             // threads per lane = 1 << log2g
+  int* err;              // device flag set on an invalid instruction
+};
+
+cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
+
+// Measured FP64 fused multiply-add throughput of the current device (flop/s, 2 per FMA).
+cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s);
+
+}  // namespace ndvm

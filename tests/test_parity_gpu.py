@@ -1,0 +1,212 @@
+"""GPU parity: the CUDA replay (through the C ABI) against the oracle, lane by lane.
+
+Tolerance (fp64): 1e-12 relative, with the rule in conftest.rel_check -- loss relative
+to |oracle loss|, each gradient component relative to the largest |component| of that
+lane's oracle gradient.  Inputs are the seeded workloads of ``workloads`` at small
+sizes (every lane checked, ragged lane counts) and at the benchmark's full sizes
+(lanes sampled and recomputed by the oracle one by one).
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+from conftest import rel_check
+
+pytestmark = pytest.mark.gpu
+
+TOL64 = 1e-12
+
+
+def gpu_run(nd, w, dtype="f64", ws_bytes=None, lanes=None):
+    import torch
+    tdt = torch.float64 if dtype == "f64" else torch.float32
+    tape = nd.trace_build(w.program, w.frontend)
+    params = w.params if lanes is None else w.params[:lanes]
+    p = torch.tensor(params, dtype=tdt, device="cuda")
+    o = torch.tensor(w.obs, dtype=tdt, device="cuda")
+    loss, grad = nd.value_and_grad(tape, p, o, ws_bytes=ws_bytes)
+    fl = nd.forward(tape, p, o)
+    torch.cuda.synchronize()
+    nd.check_device(tape)
+    return loss.double().cpu().numpy(), grad.double().cpu().numpy(), fl.double().cpu().numpy()
+
+
+def oracle_run(oracle_mod, w, idx=None, nthreads=8):
+    """(loss, grad, magnitudes) of the oracle for all lanes or the lanes idx."""
+    params = w.params if idx is None else w.params[idx]
+    return oracle_mod.run(w.program, params, w.obs, frontend=w.frontend, nthreads=nthreads, magnitudes=True)
+
+
+def check(gl, gg, ol, og, om=None, tol=TOL64):
+    ok, rep = rel_check(gl, gg, ol, og, tol, om)
+    assert ok, rep
+    return rep
+
+
+def test_exp_decay_full(ndvm, oracle_mod, cuda):
+    w = W.exp_decay()                      # B = 64 lanes, 50 points
+    gl, gg, fl = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(fl, gl)  # value-only plan gives the same bits
+
+
+@pytest.mark.parametrize("B", [1, 37, 300])
+def test_exp_decay_ragged(ndvm, oracle_mod, cuda, B):
+    w = W.exp_decay(B=B, n_points=23, seed=7)
+    gl, gg, _ = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+
+
+def test_random_exprs_small(ndvm, oracle_mod, cuda):
+    ws = W.random_exprs(n_programs=40, B=37, n_points=256, seed=1234)
+    worst = 0.0
+    for w in ws:
+        gl, gg, fl = gpu_run(ndvm, w)
+        ol, og, om = oracle_run(oracle_mod, w)
+        rep = check(gl, gg, ol, og, om)
+        worst = max(worst, rep["worst_loss"], rep["worst_grad"])
+        np.testing.assert_array_equal(fl, gl)
+    print("worst relative error", worst)
+
+
+def test_random_exprs_full_size_sampled(ndvm, oracle_mod, cuda):
+    """Full benchmark size (B = 4096 lanes, 256 points); 64 sampled lanes per program."""
+    ws = W.random_exprs(n_programs=8, B=4096, n_points=256, seed=1234)
+    rng = np.random.default_rng(0)
+    for w in ws:
+        gl, gg, _ = gpu_run(ndvm, w)
+        idx = np.sort(rng.choice(w.B, 64, replace=False))
+        ol, og, om = oracle_run(oracle_mod, w, idx)
+        check(gl[idx], gg[idx], ol, og, om)
+
+
+def test_logistic_bytecode(ndvm, oracle_mod, cuda):
+    w = W.logistic(B=200)
+    gl, gg, fl = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(fl, gl)
+
+
+def test_logistic_full_size_sampled(ndvm, oracle_mod, cuda):
+    w = W.logistic()                       # B = 16384
+    gl, gg, _ = gpu_run(ndvm, w)
+    idx = np.sort(np.random.default_rng(1).choice(w.B, 96, replace=False))
+    ol, og, om = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, om)
+
+
+def test_logistic_workspace_chunks(ndvm, oracle_mod, cuda):
+    """A workspace smaller than B lanes runs the lanes in several launches."""
+    w = W.logistic(B=1000)
+    tape = ndvm.trace_build(w.program, w.frontend)
+    per_lane = tape.workspace_bytes(1)
+    gl, gg, _ = gpu_run(ndvm, w, ws_bytes=per_lane * 300)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+
+
+def test_kalman_cv4(ndvm, oracle_mod, cuda):
+    w = W.kalman_cv4(B=70, T=200)
+    gl, gg, fl = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(fl, gl)
+
+
+def test_kalman_cv4_full_size_sampled(ndvm, oracle_mod, cuda):
+    w = W.kalman_cv4()                     # B = 8192, T = 200
+    gl, gg, _ = gpu_run(ndvm, w)
+    idx = np.sort(np.random.default_rng(2).choice(w.B, 64, replace=False))
+    ol, og, om = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, om)
+
+
+def test_kalman_rand8_short(ndvm, oracle_mod, cuda):
+    w = W.kalman_rand8(B=40, T=60)
+    gl, gg, fl = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(fl, gl)
+
+
+def test_kalman_rand8_full_T_sampled(ndvm, oracle_mod, cuda):
+    """T = 1000 steps at the full-size launch shape, on the first 1024 of the 65536 lanes."""
+    w = W.kalman_rand8()
+    gl, gg, _ = gpu_run(ndvm, w, lanes=1024)
+    idx = np.sort(np.random.default_rng(3).choice(1024, 24, replace=False))
+    ol, og, om = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, om)
+
+
+def test_lane_decomposition(ndvm, cuda):
+    """A batched run equals single-lane runs, bit for bit (section 6's lane decomposition)."""
+    for w in (W.exp_decay(B=9), W.logistic(B=9), W.kalman_cv4(B=9, T=30), W.random_exprs(2, B=9, n_points=40)[1]):
+        gl, gg, _ = gpu_run(ndvm, w)
+        for b in range(w.B):
+            one = W.Workload(w.name, w.program, w.frontend, w.params[b:b + 1], w.obs, w.truth)
+            l1, g1, _ = gpu_run(ndvm, one)
+            np.testing.assert_array_equal(l1[0], gl[b])
+            np.testing.assert_array_equal(g1[0], gg[b])
+
+
+def test_identical_lanes_identical_outputs(ndvm, cuda):
+    w = W.kalman_cv4(B=5, T=40)
+    w.params[:] = w.params[0]
+    gl, gg, _ = gpu_run(ndvm, w)
+    assert np.all(gl == gl[0]) and np.all(gg == gg[0])
+
+
+def test_repeat_runs_bit_identical(ndvm, cuda):
+    w = W.random_exprs(3, B=500, n_points=256)[2]
+    a = gpu_run(ndvm, w)
+    b = gpu_run(ndvm, w)
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
+
+
+SELECT_PROG = """
+(model (params a b)
+  (let* ((x (* a 2.0))
+         (y (if (< x 1.0) (* x b) (exp (- x b))))
+         (z (if (> b 0.0) (log (- 0.0 b)) (* b b))))
+    (+ y z (sqrt (- a 0.5)) (abs b))))
+"""
+
+
+def test_select_clamps_and_gating(ndvm, oracle_mod, cuda):
+    """Per-lane branches (lane masks) and the 1e-8 clamps of log/sqrt at their edges."""
+    rng = np.random.default_rng(5)
+    a = np.concatenate([rng.uniform(-1, 2, 60), [0.5, 0.5 + 1e-9, 0.5 + 2e-8, 0.49, 0.0]])
+    b = np.concatenate([rng.uniform(-2, 2, 60), [0.0, -1e-9, 1.0, -0.5, 0.0]])
+    w = W.Workload("select", SELECT_PROG, 0, np.stack([a, b], 1), np.zeros(0), np.zeros(2))
+    gl, gg, _ = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+
+
+def test_empty_batch_and_zero_points(ndvm, cuda):
+    import torch
+    t = ndvm.trace_build(W.exp_decay(B=1).program)
+    p = torch.zeros((0, 3), dtype=torch.float64, device="cuda")
+    o = torch.zeros(100, dtype=torch.float64, device="cuda")
+    loss, grad = ndvm.value_and_grad(t, p, o)
+    assert loss.numel() == 0 and grad.shape == (0, 3)
+    prog = "(model (params a) (+ (data-sum 0 2 (* a (dobs 0))) (* a a)))"
+    t2 = ndvm.trace_build(prog)
+    p2 = torch.tensor([[3.0], [-2.0]], dtype=torch.float64, device="cuda")
+    l2, g2 = ndvm.value_and_grad(t2, p2, None)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(l2.cpu().numpy(), [9.0, 4.0])
+    np.testing.assert_array_equal(g2.cpu().numpy(), [[6.0], [-4.0]])
+
+
+def test_host_entry_point_matches_device(ndvm, cuda):
+    w = W.logistic(B=77)
+    tape = ndvm.trace_build(w.program, w.frontend)
+    hl, hg = ndvm.value_and_grad_host(tape, w.params, w.obs)
+    gl, gg, _ = gpu_run(ndvm, w)
+    np.testing.assert_array_equal(hl, gl)
+    np.testing.assert_array_equal(hg, gg)
