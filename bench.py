@@ -44,6 +44,22 @@ def dist_env():
     return rank, world, local
 
 
+def rank_seed(rank: int) -> int:
+    """Each rank replays its own seeded population (weak scaling: per-GPU work fixed)."""
+    return SEED + 7919 * rank
+
+
+def max_over_ranks(ms: float, device=None) -> float:
+    """Step time of the whole job: the slowest rank's (no data-path collective exists)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 class ClockSampler:
     """nvidia-smi clock/throttle samples taken during the timed region."""
 
@@ -143,8 +159,10 @@ def main():
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
-    ap.add_argument("--ref-lanes", type=int, default=48, help="oracle lanes per program per reference step")
-    ap.add_argument("--cpu-lanes", type=int, default=48, help="oracle lanes per program for cpu_baseline")
+    ap.add_argument("--programs", type=int, default=N_PROGRAMS, help="programs per step (smaller for profiling)")
+    ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
+    ap.add_argument("--cpu-lanes", type=int, default=1024, help="oracle lanes per program for cpu_baseline")
+    ap.add_argument("--streams", type=int, default=4, help="CUDA streams the programs are spread over")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -164,7 +182,7 @@ def main():
     nd.load()
 
     # ---- workload: programs traced once on the host; inputs resident in HBM
-    progs = W.random_exprs(n_programs=N_PROGRAMS, B=B_LANES, n_points=N_POINTS, seed=SEED + rank)
+    progs = W.random_exprs(n_programs=args.programs, B=B_LANES, n_points=N_POINTS, seed=rank_seed(rank))
     t0 = time.perf_counter()
     tapes = [nd.trace_build(w.program, w.frontend) for w in progs]
     trace_s = time.perf_counter() - t0
@@ -179,9 +197,26 @@ def main():
         c = tp.cost()
         work += (c["work_fwd"] + c["work_rev"]) * w.B
 
+    # independent programs run on several streams so their kernels co-reside on the SMs
+    side = [torch.cuda.Stream(dev) for _ in range(args.streams)]
+
     def step():
-        for k in range(N_PROGRAMS):
-            nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=stream)
+        if args.streams <= 1:
+            for k in range(args.programs):
+                nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=stream)
+            return
+        start = torch.cuda.Event()
+        start.record(stream)
+        done = []
+        for j, s in enumerate(side):
+            s.wait_event(start)
+            for k in range(j, args.programs, args.streams):
+                nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=s)
+            e = torch.cuda.Event()
+            e.record(s)
+            done.append(e)
+        for e in done:
+            stream.wait_event(e)
 
     for _ in range(args.warmup):
         step()
@@ -207,13 +242,9 @@ def main():
     wall = time.perf_counter() - wall0
     launches = nd.launch_count() - l0
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    ms = float(np.mean(step_ms))
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(float(np.mean(step_ms)), dev)
     clk = clocks.stop()
-    lanes_per_step = N_PROGRAMS * B_LANES * world
+    lanes_per_step = args.programs * B_LANES * world
     value = lanes_per_step / (ms * 1e-3)
 
     # ---- end to end through the host-buffer entry point (pinned host memory)
@@ -223,7 +254,7 @@ def main():
     d2h = sum(w.B * 8 * (1 + w.P) for w in progs)
 
     def e2e_step():
-        for k in range(N_PROGRAMS):
+        for k in range(args.programs):
             nd.value_and_grad_host(tapes[k], hp[k], ho[k])
 
     e2e_step()
@@ -249,16 +280,16 @@ def main():
         oracle_sample_time(progs[:2], 2, cores)
         n, dt = oracle_sample_time(progs, args.cpu_lanes, cores)
         cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{args.cpu_lanes} lanes of each of the {N_PROGRAMS} programs ({n} lane evals, {dt:.1f} s)"}
+               "sample": f"{args.cpu_lanes} lanes of each of the {args.programs} programs ({n} lane evals, {dt:.1f} s)"}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "programs": N_PROGRAMS, "lanes_per_program": B_LANES,
+            "config": {"workload": WORKLOAD, "programs": args.programs, "lanes_per_program": B_LANES,
                        "points": N_POINTS, "seed": SEED, "l2": "flushed (256 MB write) before every timed step",
-                       "parallelism": f"lanes sharded, dp{world}"},
+                       "parallelism": f"lanes sharded, dp{world}", "streams": args.streams},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches // max(1, args.steps) * args.steps,
             "roofline": roofline,

@@ -64,18 +64,21 @@ class OracleError(RuntimeError):
 
 
 def run(program: str, params, obs, *, frontend: int = FRONTEND_SCHEME, mode: int = MODE_REVERSE,
-        nthreads: int = 1, magnitudes: bool = False):
+        nthreads: int = 1, magnitudes: bool = False, f32: bool = False):
     """Evaluate every lane.  params: (B, P) float64; obs: (n_obs,) float64.
 
     Returns (loss[B], grad[B, P]) (grad is None in value-only mode); with
     magnitudes=True (reverse mode) also mag[B, P], the gradient propagated through
-    absolute values -- the size of the terms each component sums.
+    absolute values -- the size of the terms each component sums.  f32=True evaluates
+    in binary32 arithmetic (each result rounded to float; inputs rounded first).
     """
     lib = _load()
     params = np.ascontiguousarray(params, dtype=np.float64)
     if params.ndim != 2:
         raise ValueError("params must be (B, P)")
     obs = np.ascontiguousarray(obs, dtype=np.float64).reshape(-1)
+    if f32:
+        obs = obs.astype(np.float32).astype(np.float64)
     B, P = params.shape
     loss = np.zeros(B, dtype=np.float64)
     grad = np.zeros((B, P), dtype=np.float64) if mode != MODE_VALUE else None
@@ -85,7 +88,8 @@ def run(program: str, params, obs, *, frontend: int = FRONTEND_SCHEME, mode: int
     rc = lib.ndvm_oracle_run(text, len(text), frontend, B, P,
                              params.ctypes.data, obs.size, obs.ctypes.data if obs.size else None,
                              loss.ctypes.data, grad.ctypes.data if grad is not None else None,
-                             mag.ctypes.data if mag is not None else None, mode, nthreads, err, len(err))
+                             mag.ctypes.data if mag is not None else None, mode | (4 if f32 else 0), nthreads,
+                             err, len(err))
     if rc != 0:
         raise OracleError(err.value.decode(errors="replace"))
     if magnitudes:

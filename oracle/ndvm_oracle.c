@@ -149,7 +149,7 @@ typedef struct {
 typedef struct {
   const Program* prog;
   Arena* ar;
-  int mode, P;
+  int mode, P, f32;  /* f32: round every arithmetic result to binary32 */
   const double* theta;     /* this lane's parameters */
   const double* obs; long long nobs;
   /* data-axis context for (dobs k) */
@@ -159,6 +159,10 @@ typedef struct {
   char* err; size_t errcap;
   int depth;
 } Ctx;
+
+/* fp32 mode: a result computed in double and rounded once to float is the correctly
+ * rounded float result for + - * / and sqrt (53 >= 2*24 + 2 bits). */
+#define RF(cx, x) ((cx)->f32 ? (double)(float)(x) : (x))
 
 static void fail(Ctx* cx, const char* fmt, ...) {
   va_list ap; va_start(ap, fmt);
@@ -348,7 +352,7 @@ static int any_dep(Num* n) {
 }
 static Num* const_num(Ctx* cx, double x) {
   Num* n = new_num(cx, N_CONST, 1, 1, 0);
-  n->v[0] = x; return n;
+  n->v[0] = RF(cx, x); return n;
 }
 static int is_scalar(Num* n) { return n->r == 1 && n->c == 1; }
 
@@ -372,7 +376,7 @@ static Num* unary(Ctx* cx, int kind, Num* x) {
     case N_ABS: v = fabs(a); dv = (a > 0) ? 1.0 : (a < 0 ? -1.0 : 0.0); break;
     default: fail(cx, "internal: bad unary kind");
   }
-  z->v[0] = v;
+  z->v[0] = RF(cx, v);
   if (cx->mode == MODE_DUAL && x->d) {
     dual_alloc(cx, z);
     for (int k = 0; k < cx->P; k++) z->d[k] = dv * x->d[k];
@@ -387,16 +391,16 @@ static Num* nary(Ctx* cx, int kind, int n, Num** xs) {
   for (int i = 0; i < n; i++) z->in[i] = xs[i];
   z->dep = any_dep(z);
   double v = 0;
-  if (kind == N_ADD) { v = xs[0]->v[0]; for (int i = 1; i < n; i++) v = v + xs[i]->v[0]; }
+  if (kind == N_ADD) { v = xs[0]->v[0]; for (int i = 1; i < n; i++) v = RF(cx, v + xs[i]->v[0]); }
   else if (kind == N_SUB) {
     if (n == 1) v = -xs[0]->v[0];
-    else { double s = xs[1]->v[0]; for (int i = 2; i < n; i++) s = s + xs[i]->v[0]; v = xs[0]->v[0] - s; }
-  } else if (kind == N_MUL) { v = xs[0]->v[0]; for (int i = 1; i < n; i++) v = v * xs[i]->v[0]; }
+    else { double s = xs[1]->v[0]; for (int i = 2; i < n; i++) s = RF(cx, s + xs[i]->v[0]); v = xs[0]->v[0] - s; }
+  } else if (kind == N_MUL) { v = xs[0]->v[0]; for (int i = 1; i < n; i++) v = RF(cx, v * xs[i]->v[0]); }
   else if (kind == N_DIV) {
     if (n == 1) v = 1.0 / xs[0]->v[0];
-    else { double p = xs[1]->v[0]; for (int i = 2; i < n; i++) p = p * xs[i]->v[0]; v = xs[0]->v[0] / p; }
+    else { double p = xs[1]->v[0]; for (int i = 2; i < n; i++) p = RF(cx, p * xs[i]->v[0]); v = xs[0]->v[0] / p; }
   }
-  z->v[0] = v;
+  z->v[0] = RF(cx, v);
   if (cx->mode == MODE_DUAL && z->dep) {
     dual_alloc(cx, z);
     for (int k = 0; k < cx->P; k++) {
@@ -500,7 +504,7 @@ static Num* mat_from(Ctx* cx, int r, int c, Num** el) {
 }
 static Num* const_mat(Ctx* cx, int r, int c, const double* v) {
   Num* z = new_num(cx, N_CONST, r, c, 0);
-  memcpy(z->v, v, sizeof(double) * r * c);
+  for (int i = 0; i < r * c; i++) z->v[i] = RF(cx, v[i]);
   return z;
 }
 static Num* mref_num(Ctx* cx, Num* a, long long i, long long j) {
@@ -739,8 +743,8 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
   gbuf_sel(cx, loss, absmode)[0] = 1.0;
 #define gbuf(cx, x) gbuf_sel(cx, x, absmode)
 #define F(v) (absmode ? fabs(v) : (v))
-#define ADD(dst, v) ((dst) += (absmode ? fabs(v) : (v)))
-#define SUB(dst, v) ((dst) += (absmode ? fabs(v) : -(v)))
+#define ADD(dst, v) ((dst) = RF(cx, (dst) + (absmode ? fabs(v) : RF(cx, (v)))))
+#define SUB(dst, v) ((dst) = RF(cx, (dst) + (absmode ? fabs(v) : -RF(cx, (v)))))
   for (size_t q = cnt; q-- > 0;) {
     Num* n = order[q];
     size_t m = (size_t)n->r * n->c;
@@ -1464,6 +1468,7 @@ typedef struct {
   double* loss; double* grad; double* mag;
   long long b0, b1;
   int status; char err[512];
+  int f32;
 } Job;
 
 /* One lane: evaluate, then differentiate; errors unwind here. */
@@ -1471,7 +1476,14 @@ static int run_lane(Job* jb, Arena* ar, long long b, double* g) {
   Ctx cx;
   memset(&cx, 0, sizeof(cx));
   cx.prog = jb->prog; cx.ar = ar; cx.mode = jb->mode; cx.P = jb->P;
+  cx.f32 = jb->f32;
+  double theta32[64];
   cx.theta = jb->params + b * jb->P; cx.obs = jb->obs; cx.nobs = jb->nobs;
+  if (jb->f32) {  /* parameters rounded to float (observations are rounded by the caller) */
+    if (jb->P > 64) { snprintf(jb->err, sizeof(jb->err), "fp32 mode supports at most 64 parameters"); return OR_ERR; }
+    for (int k = 0; k < jb->P; k++) theta32[k] = (double)(float)cx.theta[k];
+    cx.theta = theta32;
+  }
   cx.err = jb->err; cx.errcap = sizeof(jb->err);
   if (setjmp(cx.jb)) return OR_ERR;
   Num* loss = jb->frontend == 0 ? run_scheme(&cx) : run_bytecode(&cx);
@@ -1520,7 +1532,9 @@ static void free_program(Program* pg) {
  *   loss        : B outputs; grad: B x P outputs or NULL
  *   mag         : B x P magnitude scales (reverse mode only) or NULL: the gradient
  *                 propagated through absolute values, bounding the terms summed
- *   mode        : 0 value only, 1 reverse mode, 2 dual numbers
+ *   mode        : 0 value only, 1 reverse mode, 2 dual numbers; + 4 = fp32 mode
+ *                 (every arithmetic result rounded to binary32; obs must be
+ *                 given already rounded to float)
  *   nthreads    : worker threads (lanes split into contiguous chunks)
  * Returns 0 on success; on error writes a message into err.
  */
@@ -1529,6 +1543,8 @@ int ndvm_oracle_run(const char* program, size_t len, int frontend, long long B, 
                     double* loss, double* grad, double* mag, int mode, int nthreads, char* err, size_t errcap) {
   Program pg; memset(&pg, 0, sizeof(pg));
   if (err && errcap) err[0] = 0;
+  const int f32 = (mode & 4) != 0;
+  mode &= 3;
   if (B < 0 || P < 0 || (frontend != 0 && frontend != 1) || mode < 0 || mode > 2) {
     if (err) snprintf(err, errcap, "bad arguments");
     return OR_ERR;
@@ -1556,7 +1572,7 @@ int ndvm_oracle_run(const char* program, size_t len, int frontend, long long B, 
   long long per = (B + nthreads - 1) / (nthreads ? nthreads : 1);
   for (int t = 0; t < nthreads; t++) {
     Job* j = &jobs[t];
-    j->prog = &pg; j->frontend = frontend; j->mode = mode; j->P = P;
+    j->prog = &pg; j->frontend = frontend; j->mode = mode; j->P = P; j->f32 = f32;
     j->params = params; j->obs = obs; j->nobs = nobs; j->loss = loss; j->grad = grad; j->mag = mag;
     j->b0 = t * per; j->b1 = (t + 1) * per < B ? (t + 1) * per : B;
     if (j->b0 > B) j->b0 = B;

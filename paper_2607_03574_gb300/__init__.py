@@ -212,7 +212,7 @@ class Workspace:
         return self.buf
 
 
-_default_ws = Workspace()
+_default_ws = {}  # (device, stream) -> Workspace: concurrent streams never share one
 
 
 def value_and_grad(tape: Tape, params, obs, loss=None, grad=None, workspace=None, ws_bytes=None, stream=None):
@@ -226,7 +226,8 @@ def value_and_grad(tape: Tape, params, obs, loss=None, grad=None, workspace=None
     dt = _dtype_code(params)
     if workspace is None:
         need = tape.workspace_bytes(B, dt) if ws_bytes is None else ws_bytes
-        workspace = _default_ws.get(need, params.device)
+        key = (str(params.device), _stream_ptr(stream).value)
+        workspace = _default_ws.setdefault(key, Workspace()).get(need, params.device)
     nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     if ws_bytes is not None:
         nbytes = min(nbytes, ws_bytes)

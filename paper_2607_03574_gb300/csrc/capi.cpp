@@ -2,6 +2,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -53,7 +54,8 @@ struct DevCache {
 struct ndvm_tape {
   Tape tape;
   Plan grad_plan, value_plan;
-  std::mutex mu;
+  std::mutex mu;       // guards dev (device copies)
+  std::mutex host_mu;  // serializes the host-buffer entry point and its cached buffers
   std::map<int, DevCache> dev;
 };
 
@@ -111,14 +113,29 @@ ndvm_status device_cache(ndvm_tape* t, DevCache** out) {
 
 constexpr size_t kSmemLimit = 227 * 1024;
 
+// Threads per lane for data-axis tapes: NDVM_THREADS_PER_LANE (1..32, a power of two)
+// overrides the default, which splits a lane's points over enough threads to give
+// the launch about 512 threads per SM.
+int threads_per_lane_override() {
+  static int v = [] {
+    const char* e = std::getenv("NDVM_THREADS_PER_LANE");
+    int g = e ? std::atoi(e) : 0;
+    return (g >= 1 && g <= 32 && (g & (g - 1)) == 0) ? g : 0;
+  }();
+  return v;
+}
+
 // threads per block and threads per lane for a plan
 void launch_shape(const Plan& p, size_t elem, int64_t B, int& tpb, int& log2g) {
   log2g = 0;
   if (p.has_regions && p.n_save == 0) {
     // split the data axis over a group of threads when lanes alone cannot fill the GPU
-    const int64_t target = 152LL * 1024;
-    int g = 1;
-    while (g < 32 && B * g < target) g *= 2;
+    const int64_t target = 152LL * 512;
+    int g = threads_per_lane_override();
+    if (!g) {
+      g = 1;
+      while (g < 32 && B * g < target) g *= 2;
+    }
     while ((1 << log2g) < g) log2g++;
   }
   tpb = 128;
@@ -314,7 +331,7 @@ ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, in
   const size_t pb = (size_t)B * t->tape.n_params * elem, ob = (size_t)n_obs * elem, lb = (size_t)B * elem;
   const bool want_grad = grad != nullptr;
   size_t wsb = want_grad ? ndvm_workspace_bytes(t, B, dtype) : 0;
-  std::lock_guard<std::mutex> lk(t->mu);
+  std::lock_guard<std::mutex> lk(t->host_mu);
   if ((s = ensure(&dc->h_params, &dc->h_params_bytes, pb)) != NDVM_OK) return s;
   if ((s = ensure(&dc->h_obs, &dc->h_obs_bytes, ob)) != NDVM_OK) return s;
   if ((s = ensure(&dc->h_loss, &dc->h_loss_bytes, lb)) != NDVM_OK) return s;

@@ -1,20 +1,20 @@
 // Algorithmic FP64 work per tape primitive, in DFMA-equivalents (one fused
 // multiply-add issue of the FP64 pipe = 1).  Arithmetic counts one per add,
 // multiply or fused multiply-add; a first adjoint contribution that is a copy or a
-// sign flip counts zero.  Library functions count their throughput cost relative
-// to DFMA, measured on GB300 for CUDA's double-precision functions with many
-// independent calls per thread (exp 17.6, log 28.7, sin or cos 17.4, sincos 22.7,
-// tanh 13.7, sqrt 7.5, reciprocal 4.6, pow 85).  The roofline divides this work by
-// the measured DFMA rate.
+// sign flip counts zero.  Functions count their throughput cost relative to DFMA,
+// measured on GB300 with many independent calls per thread on finite arguments:
+// the replay's own exp 9.7 and log 12.6 (fmath.cuh), and CUDA's sin 17.1,
+// sincos 22.3, tanh 13.5, sqrt 7.3, division 7.1, reciprocal 4.4, log 28.5 (inside
+// pow's adjoint) and pow 79.9.  The roofline divides this work by the measured
+// DFMA rate.
 #pragma once
 #include "tape.h"
 
 namespace ndvm {
 namespace cost {
 
-constexpr double kExp = 17.6, kLog = 28.7, kSin = 17.4, kSinCos = 22.7, kTanh = 13.7, kSqrt = 7.5,
-                 kRcp = 4.6, kPow = 85.0;
-constexpr double kDiv = kRcp + 1.0;
+constexpr double kExp = 9.7, kLog = 12.6, kSin = 17.1, kSinCos = 22.3, kTanh = 13.5, kSqrt = 7.3,
+                 kRcp = 4.4, kPow = 79.9, kDiv = 7.1, kLogLib = 28.5;
 
 inline double inv_cost(int n) {
   if (n == 1) return kDiv;
@@ -62,7 +62,7 @@ inline double rev(int op, int r, int c, int imm, int n, bool aa, bool ba, bool a
     case OP_NEG: return acc(aa, a_init);
     case OP_MUL: return (aa ? 1 : 0) + (ba ? 1 : 0);
     case OP_DIV: return kDiv + acc(aa, a_init) + (ba ? 1 : 0);
-    case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLog + 2 : 0);
+    case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLogLib + 2 : 0);
     case OP_EXP: case OP_SIN: case OP_COS: case OP_ABS: return 1;
     case OP_TANH: return 2;
     case OP_LOG: return kDiv + 1;

@@ -125,8 +125,18 @@ void Planner::analyze() {
   for (int v = 0; v < N; v++) {
     const Node& n = T.nodes[v];
     if (n.op == OP_DSUM) {
-      for (int u = n.a; u < n.b; u++) region_body_[u] = 1;
-      if (n.c >= n.a && n.c < n.b) {} else if (n.c >= v) unsupported("malformed data-sum");
+      // Only nodes that depend on the data point run per point; a node traced
+      // inside the body but independent of the point is hoisted: it runs once per
+      // lane, and its adjoint arrives through the region's partial sums.
+      if (n.a < 0 || n.b > v || n.a > n.b) unsupported("malformed data-sum");
+      for (int u = n.a; u < n.b; u++) {
+        const Node& m = T.nodes[u];
+        if (m.op == OP_DOBS) { region_body_[u] = 1; continue; }
+        if (m.op == OP_CONST || m.op == OP_PARAM || m.op == OP_OBS) continue;
+        for (int x : inputs(u))
+          if (x >= n.a && x < u && region_body_[x]) { region_body_[u] = 1; break; }
+      }
+      if (n.c >= v) unsupported("malformed data-sum");
     }
   }
   for (int v = 0; v < N; v++) {
@@ -443,7 +453,7 @@ void Planner::emit_reverse(int v) {
 void Planner::emit_region(int v) {
   const Node& n = T.nodes[v];
   const int b0 = n.a, b1 = n.b, res = n.c;
-  auto body_value = [&](int x) { return x >= b0 && x < b1 && !is_leaf(x); };
+  auto body_value = [&](int x) { return x >= b0 && x < b1 && region_body_[x] && !is_leaf(x); };
   // lane-level inputs whose partials the body reverse accumulates
   std::vector<std::pair<int, int>> ins;
   std::vector<char> seen(N, 0);
@@ -454,7 +464,7 @@ void Planner::emit_region(int v) {
   };
   if (grad_) {
     for (int u = b0; u < b1; u++) {
-      if (is_leaf(u) || !active_[u]) continue;
+      if (!body_value(u) || !active_[u]) continue;
       const Node& m = T.nodes[u];
       if (m.op == OP_SELECT) { add_input(m.b); add_input(m.c); continue; }
       for (int x : inputs(u)) add_input(x);
@@ -474,7 +484,7 @@ void Planner::emit_region(int v) {
   mult_ = (double)n.imm;
   work_fwd_ += mult_;  // accumulation of the body value
   for (int u = b0; u < b1; u++) {
-    if (is_leaf(u)) continue;
+    if (!body_value(u)) continue;
     if (T.nodes[u].op == OP_DSUM) unsupported("nested data-sum");
     emit_forward(u);
   }
@@ -495,7 +505,7 @@ void Planner::emit_region(int v) {
       emit(a1);
     }
     for (int u = b1 - 1; u >= b0; u--) {
-      if (is_leaf(u) || !active_[u]) continue;
+      if (!body_value(u) || !active_[u]) continue;
       emit_reverse(u);
     }
     for (auto& io : ins) partial_of_[io.first] = -1;

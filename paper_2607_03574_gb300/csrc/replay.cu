@@ -23,6 +23,7 @@
 
 #include "plan.h"
 #include "replay.h"
+#include "fmath.cuh"
 
 namespace ndvm {
 namespace {
@@ -73,6 +74,19 @@ struct Lane {
 };
 
 template <typename T> __device__ __forceinline__ T clamp_eps() { return (T)1e-8; }
+
+// Tests on IEEE bit patterns run on the integer pipes, leaving the FP64 pipe to
+// arithmetic.  is_zero: +0 or -0.  gt_eps: x > 1e-8 with NaN false (IEEE order).
+__device__ __forceinline__ bool is_zero(double x) { return (__double_as_longlong(x) << 1) == 0; }
+__device__ __forceinline__ bool is_zero(float x) { return (__float_as_uint(x) << 1) == 0u; }
+__device__ __forceinline__ bool gt_eps(double x) {
+  const long long b = __double_as_longlong(x);
+  return b > __double_as_longlong(1e-8) && (b & 0x7fffffffffffffffLL) <= 0x7ff0000000000000LL;
+}
+__device__ __forceinline__ bool gt_eps(float x) {
+  const int b = __float_as_int(x);
+  return b > __float_as_int(1e-8f) && (b & 0x7fffffff) <= 0x7f800000;
+}
 
 template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
   if (n == 0) return (T)1;
@@ -155,7 +169,7 @@ __device__ T det_inv(const Opnd<T>& A, int n, T* inv /* n*n or nullptr */) {
 template <typename T>
 __device__ __forceinline__ bool all_zero(const Lane<T>& L, int32_t gz, int w) {
   for (int e = 0; e < w; e++)
-    if (L.sl(gz, e) != (T)0) return false;
+    if (!is_zero(L.sl(gz, e))) return false;
   return true;
 }
 template <typename T>
@@ -217,10 +231,10 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: {
         T x = L.ld(f[1]), z;
         if (in.op == D_NEG) z = -x;
-        else if (in.op == D_EXP) z = exp(x);
-        else if (in.op == D_LOG) z = log(x > clamp_eps<T>() ? x : clamp_eps<T>());
+        else if (in.op == D_EXP) z = fast_exp(x);
+        else if (in.op == D_LOG) z = fast_log(gt_eps(x) ? x : clamp_eps<T>());
         else if (in.op == D_TANH) z = tanh(x);
-        else if (in.op == D_SQRT) z = sqrt(x > clamp_eps<T>() ? x : clamp_eps<T>());
+        else if (in.op == D_SQRT) z = sqrt(gt_eps(x) ? x : clamp_eps<T>());
         else z = fabs(x);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
@@ -260,7 +274,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       case D_SELECT: {
         T p = L.ld(f[1]);
-        T z = p != (T)0 ? L.ld(f[2]) : L.ld(f[4]);
+        T z = !is_zero(p) ? L.ld(f[2]) : L.ld(f[4]);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
         break;
@@ -320,7 +334,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         const bool aux = f[4] != -1 || f[5] >= 0;
         T inv[64];
         T dt = det_inv(L.rd(f[1]), n, aux ? inv : nullptr);
-        T z = in.op == D_DET ? dt : log(dt);
+        T z = in.op == D_DET ? dt : fast_log(dt);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
         if (aux)
@@ -372,7 +386,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_ADD: case B_SUB: case B_NEG: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); if (in.op != B_NEG) zero_if_first(L, f[2], 1, fb); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); if (in.op != B_NEG) zero_if_first(L, f[2], 1, fb); break; }
         if (f[1] != -1) L.upd(f[1], 0, in.op == B_NEG ? -g : g, fa);
         if (in.op != B_NEG && f[2] != -1) L.upd(f[2], 0, in.op == B_ADD ? g : -g, fb);
         break;
@@ -380,7 +394,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_MUL: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
         if (f[1] != -1) L.upd(f[1], 0, g * L.ld(f[4]), fa);
         if (f[2] != -1) L.upd(f[2], 0, g * L.ld(f[3]), fb);
         break;
@@ -388,7 +402,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_DIV: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
         T q = g / L.ld(f[4]);
         if (f[1] != -1) L.upd(f[1], 0, q, fa);
         if (f[2] != -1) L.upd(f[2], 0, -(q * L.ld(f[5])), fb);
@@ -397,7 +411,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_POW: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
         T x = L.ld(f[3]), e = L.ld(f[4]), z = L.ld(f[5]);
         if (f[1] != -1) L.upd(f[1], 0, g * e * z / x, fa);
         if (f[2] != -1) L.upd(f[2], 0, g * z * log(x), fb);
@@ -407,14 +421,14 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1;
         if (f[1] == -1) break;
-        if (g == (T)0) { zero_if_first(L, f[1], 1, fa); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); break; }
         T v;
         switch (in.op) {
           case B_EXP: v = g * L.ld(f[5]); break;
           case B_TANH: { T z = L.ld(f[5]); v = g * ((T)1 - z * z); break; }
-          case B_LOG: { T x = L.ld(f[3]); v = x > clamp_eps<T>() ? g / x : (T)0; break; }
+          case B_LOG: { T x = L.ld(f[3]); v = gt_eps(x) ? g / x : (T)0; break; }
           case B_ABS: { T x = L.ld(f[3]); v = x > (T)0 ? g : (x < (T)0 ? -g : g * (T)0); break; }
-          case B_SQRT: { T x = L.ld(f[3]); v = x > clamp_eps<T>() ? g / ((T)2 * L.ld(f[5])) : (T)0; break; }
+          case B_SQRT: { T x = L.ld(f[3]); v = gt_eps(x) ? g / ((T)2 * L.ld(f[5])) : (T)0; break; }
           case B_SIN: v = g * L.ld(f[6]); break;
           case B_COS: v = -(g * L.ld(f[6])); break;
           default: {  // POWI
@@ -428,9 +442,9 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_SELECT: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        bool taken = L.ld(f[3]) != (T)0;
-        if (f[1] != -1) { if (taken && g != (T)0) L.upd(f[1], 0, g, fa); else zero_if_first(L, f[1], 1, fa); }
-        if (f[2] != -1) { if (!taken && g != (T)0) L.upd(f[2], 0, g, fb); else zero_if_first(L, f[2], 1, fb); }
+        bool taken = !is_zero(L.ld(f[3]));
+        if (f[1] != -1) { if (taken && !is_zero(g)) L.upd(f[1], 0, g, fa); else zero_if_first(L, f[1], 1, fa); }
+        if (f[2] != -1) { if (!taken && !is_zero(g)) L.upd(f[2], 0, g, fb); else zero_if_first(L, f[2], 1, fb); }
         break;
       }
       case B_GATHER: {
@@ -531,7 +545,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         bool fa = in.flags & 1;
         if (f[1] == -1) break;
         T g = L.sl(f[0], 0);
-        if (g == (T)0) { zero_if_first(L, f[1], n * n, fa); break; }
+        if (is_zero(g)) { zero_if_first(L, f[1], n * n, fa); break; }
         T fac = in.op == B_DET ? g * L.ld(f[5]) : g;
         Opnd<T> Iv = L.rd(f[6]);
         for (int i = 0; i < n; i++)
@@ -544,7 +558,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         if (f[1] == -1) break;
         T g = L.sl(f[0], 0);
         zero_if_first(L, f[1], n * n, fa);
-        if (g == (T)0) break;
+        if (is_zero(g)) break;
         for (int i = 0; i < n; i++) L.st(f[1], i * n + i, L.sl(f[1], i * n + i) + g);
         break;
       }
@@ -554,7 +568,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         for (int e = 0; e < f[2]; e++) {
           int32_t t = q[3 * e];
           bool first = q[3 * e + 1] != 0;
-          if (g == (T)0) zero_if_first(L, t, 1, first);
+          if (is_zero(g)) zero_if_first(L, t, 1, first);
           else L.upd(t, 0, g * L.sl(q[3 * e + 2], 0), first);
         }
         break;

@@ -422,3 +422,19 @@ def test_errors_are_reported(oracle_mod):
         run(oracle_mod, "(model (params a) (matmul (identity 2) (identity 3)))", [[1.0]])
     with pytest.raises(oracle_mod.OracleError):
         run(oracle_mod, "PARAM 0\nADD\n", [[1.0]], frontend=1)
+
+
+def test_fp32_mode_is_binary32_arithmetic(oracle_mod):
+    # every result rounded to float: identical to numpy float32 arithmetic step by step
+    P = "(model (params a b) (- (/ (+ a 0.1) (* b 3.0)) (* a a)))"
+    th = np.array([[0.7, 1.3], [-2.5, 0.11]])
+    l, g = oracle_mod.run(P, th, np.zeros(0), f32=True)
+    f = np.float32
+    for b in range(2):
+        a, bb = f(th[b, 0]), f(th[b, 1])
+        ref = (a + f(0.1)) / (bb * f(3.0)) - a * a
+        assert l[b] == float(ref)
+    bc = "PARAM 0\nOBS 0\nADD\nPUSH 0.3\nMUL\n"
+    l, g = oracle_mod.run(bc, np.array([[0.1]]), np.array([0.2]), frontend=1, f32=True)
+    assert l[0] == float((f(0.1) + f(0.2)) * f(0.3))
+    assert g[0, 0] == float(f(0.3))

@@ -210,3 +210,22 @@ def test_host_entry_point_matches_device(ndvm, cuda):
     gl, gg, _ = gpu_run(ndvm, w)
     np.testing.assert_array_equal(hl, gl)
     np.testing.assert_array_equal(hg, gg)
+
+
+def test_logistic_fp32_variant(ndvm, oracle_mod, cuda):
+    """fp32 replay against the oracle in binary32 arithmetic, 1e-5 relative."""
+    w = W.logistic(B=300)
+    w.params = w.params.astype(np.float32).astype(np.float64)
+    gl, gg, fl = gpu_run(ndvm, w, dtype="f32")
+    ol, og, om = oracle_mod.run(w.program, w.params, w.obs, frontend=w.frontend, nthreads=8, magnitudes=True,
+                                f32=True)
+    check(gl, gg, ol, og, om, tol=1e-5)
+    np.testing.assert_array_equal(fl, gl)
+
+
+def test_exp_decay_fp32_variant(ndvm, oracle_mod, cuda):
+    w = W.exp_decay(B=64)
+    w.params = w.params.astype(np.float32).astype(np.float64)
+    gl, gg, _ = gpu_run(ndvm, w, dtype="f32")
+    ol, og, om = oracle_mod.run(w.program, w.params, w.obs, nthreads=8, magnitudes=True, f32=True)
+    check(gl, gg, ol, og, om, tol=1e-5)
