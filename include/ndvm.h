@@ -133,6 +133,29 @@ ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, in
                                      const void* obs, int64_t n_obs, void* loss, void* grad, void* stream);
 
 /*
+ * ndvm_value_and_grad_noalloc -- ndvm_value_and_grad for callers that may not
+ * allocate device memory while they run (their device memory is planned up front
+ * and must not grow).  The paper has no counterpart; this is a deployment variant.
+ * Arguments as ndvm_value_and_grad, without a workspace: the forward values that
+ * the reverse sweep reads go to a fixed scratch array of 32 MiB inside the
+ * library, held by every GPU that loads the library until the process exits.
+ * The call allocates nothing: it makes no cudaMalloc, cudaFree or other allocating
+ * call.  Therefore:
+ *   - the tape must already be resident on the current device: one earlier
+ *     ndvm_forward or ndvm_value_and_grad call for this tape uploads it (that
+ *     call allocates); otherwise NDVM_E_INVALID_ARG;
+ *   - the first call on a device looks up the scratch array's device address
+ *     (once per device); make that first call before any stream capture;
+ *   - lanes run in chunks that fit the scratch; a tape whose workspace for one
+ *     block of lanes exceeds 32 MiB is rejected with NDVM_E_INVALID_ARG;
+ *   - every call shares the one array, so calls whose work overlaps on the GPU
+ *     race; nothing in the array needs clearing (each saved value is written
+ *     before it is read).
+ */
+ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                        const void* obs, int64_t n_obs, void* loss, void* grad, void* stream);
+
+/*
  * ndvm_check_device -- synchronize and report whether any kernel of this tape
  * on the current device recorded a consistency failure (NDVM_E_DEVICE_CHECK);
  * clears the flag.

@@ -62,6 +62,7 @@ def load(build_if_missing: bool = True):
             "ndvm_forward": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P]),
             "ndvm_value_and_grad": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P, SZ, P]),
             "ndvm_value_and_grad_host": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
+            "ndvm_value_and_grad_noalloc": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_check_device": (ctypes.c_int, [P]),
             "ndvm_launch_count": (ctypes.c_ulonglong, []),
             "ndvm_measure_fp64_peak": (ctypes.c_int, [ctypes.POINTER(ctypes.c_double), P]),
@@ -235,6 +236,17 @@ def value_and_grad(tape: Tape, params, obs, loss=None, grad=None, workspace=None
                                       0 if obs is None else obs.numel(), _dev_ptr(loss, "loss"),
                                       _dev_ptr(grad, "grad"), _dev_ptr(workspace, "workspace"), nbytes,
                                       _stream_ptr(stream)))
+    return loss, grad
+
+
+def value_and_grad_noalloc(tape: Tape, params, obs, loss, grad, stream=None):
+    """Loss and gradient into caller-given outputs with no device allocation (the
+    library's fixed scratch array serves as workspace; the tape must already be
+    resident on the device)."""
+    _check(load().ndvm_value_and_grad_noalloc(tape.handle, _dtype_code(params), params.shape[0],
+                                              _dev_ptr(params, "params"), _dev_ptr(obs, "obs"),
+                                              0 if obs is None else obs.numel(), _dev_ptr(loss, "loss"),
+                                              _dev_ptr(grad, "grad"), _stream_ptr(stream)))
     return loss, grad
 
 

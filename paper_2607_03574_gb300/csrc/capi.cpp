@@ -385,4 +385,80 @@ const char* ndvm_last_error(void) { return g_last_error.c_str(); }
 
 const char* ndvm_version(void) { return "ndvm-gb300 0.1"; }
 
+// Value and gradient without allocating: the workspace is the library's fixed
+// scratch array (replay.cu) instead of caller memory, and the tape must already be
+// resident on the current device.  No cudaMalloc, cudaFree or other allocating
+// call is made here.
+ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                        const void* obs, int64_t n_obs, void* loss, void* grad, void* stream) {
+  ndvm_tape* t = const_cast<ndvm_tape*>(tape);
+  if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
+  if (dtype != NDVM_F64 && dtype != NDVM_F32) return fail(NDVM_E_INVALID_ARG, "bad dtype");
+  if (B < 0) return fail(NDVM_E_INVALID_ARG, "B must be >= 0");
+  if (B == 0) return NDVM_OK;
+  const Plan& p = t->grad_plan;
+  if (p.n_params > 0 && (!params || !grad)) return fail(NDVM_E_INVALID_ARG, "null params or grad");
+  if (!loss) return fail(NDVM_E_INVALID_ARG, "null loss");
+  if (n_obs < p.n_obs_min) return fail(NDVM_E_INVALID_ARG, "obs holds fewer values than the program reads");
+  if (p.n_obs_min > 0 && !obs) return fail(NDVM_E_INVALID_ARG, "null obs");
+  const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  int tpb, log2g;
+  launch_shape(p, elem, B, tpb, log2g);
+  const size_t smem = (size_t)p.n_slots * tpb * elem;
+  if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs more slots per lane than shared memory holds");
+  const int lanes_per_block = tpb >> log2g;
+  int64_t chunk = B;
+  if (p.n_save > 0) {
+    const size_t per_lane = (size_t)p.n_save * elem;
+    const size_t per_block = per_lane * lanes_per_block;
+    if (per_block > kNoAllocScratchBytes)
+      return fail(NDVM_E_INVALID_ARG, "this tape needs " + std::to_string(per_block) + " bytes of workspace per block of " +
+                                          std::to_string(lanes_per_block) + " lanes; the fixed scratch holds " +
+                                          std::to_string(kNoAllocScratchBytes) + " bytes");
+    int64_t fit = (int64_t)(kNoAllocScratchBytes / per_lane);
+    if (fit < B) chunk = fit - fit % lanes_per_block;
+  }
+  DevCache* dc = nullptr;
+  {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    std::lock_guard<std::mutex> lk(t->mu);
+    auto it = t->dev.find(dev);
+    if (it == t->dev.end())
+      return fail(NDVM_E_INVALID_ARG, "tape is not resident on this device; one ndvm_forward or ndvm_value_and_grad "
+                                      "call uploads it (that call allocates)");
+    dc = &it->second;
+  }
+  void* scratch = nullptr;
+  cudaError_t e = noalloc_scratch(&scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+  ReplayArgs a;
+  a.code = dc->grad.code;
+  a.n_code = (int)p.code.size();
+  a.args = dc->grad.args;
+  a.consts = dtype == NDVM_F32 ? (const void*)dc->grad.consts_f : (const void*)dc->grad.consts_d;
+  a.obs = obs;
+  a.params = params;
+  a.loss = loss;
+  a.grad = grad;
+  a.save = scratch;
+  a.save_ld = chunk;
+  a.P = p.n_params;
+  a.log2g = log2g;
+  a.err = dc->err;
+  for (int64_t l0 = 0; l0 < B; l0 += chunk) {
+    a.lane0 = l0;
+    a.lane_end = l0 + chunk < B ? l0 + chunk : B;
+    const int64_t blocks = (a.lane_end - l0 + lanes_per_block - 1) / lanes_per_block;
+    {
+      std::lock_guard<std::mutex> lk(g_launch_mu);
+      e = launch_replay(a, dtype == NDVM_F32, (int)blocks, tpb, smem, (cudaStream_t)stream);
+      g_launches++;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "replay launch");
+  }
+  return NDVM_OK;
+}
+
 }  // extern "C"

@@ -20,6 +20,8 @@
 
 #include <cmath>
 #include <cstdint>
+#include <map>
+#include <mutex>
 
 #include "plan.h"
 #include "replay.h"
@@ -658,5 +660,39 @@ cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s) {
   cudaFree(out);
   if (e == cudaSuccess) *flops_per_s = 2.0 * 8.0 * iters * (double)blocks * threads / (best * 1e-3);
   return e;
+}
+}  // namespace ndvm
+
+// ---------------------------------------------------------------------------
+// Fixed scratch for the no-allocation entry point (ndvm_value_and_grad_noalloc).
+// Some callers may not allocate device memory while they run -- their device
+// memory is planned up front and must not grow.  For them the workspace of the
+// replay lives in this file-scope array, held by every GPU that loads the
+// library until the process exits.  Every call uses the same array, so calls
+// whose work overlaps on the GPU race; the replay writes each saved element
+// before it reads it, so nothing in it needs clearing between calls.
+namespace ndvm {
+namespace {
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+}  // namespace
+
+cudaError_t noalloc_scratch(void** ptr) {
+  // The array's name is a host-side stand-in; its device address is looked up
+  // once per device, with that device current.
+  static std::mutex mu;
+  static std::map<int, void*> addr;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = addr.find(dev);
+  if (it == addr.end()) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    it = addr.emplace(dev, p).first;
+  }
+  *ptr = it->second;
+  return cudaSuccess;
 }
 }  // namespace ndvm

@@ -28,6 +28,12 @@ struct ReplayArgs {
 
 cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
 
+// Size of the fixed scratch array of the no-allocation entry point (32 MiB).
+constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;
+
+// Device address of that array on the current device (looked up once per device).
+cudaError_t noalloc_scratch(void** ptr);
+
 // Measured FP64 fused multiply-add throughput of the current device (flop/s, 2 per FMA).
 cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s);
 

@@ -1,0 +1,71 @@
+"""The no-allocation entry point, checked against the regular one (GPU).
+
+ndvm_value_and_grad_noalloc is for callers that may not allocate device memory while
+they run -- a service whose device memory is planned up front and must not grow, or a
+host runtime that owns every allocation.  It allocates nothing: the replay's workspace
+is a fixed 32 MiB scratch array inside the library, and the tape must already be
+resident on the device.  These tests call it through the C ABI and compare it with
+ndvm_value_and_grad, twice in a row (the array keeps the previous call's contents).
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+import workloads as W
+from conftest import rel_check
+
+pytestmark = pytest.mark.gpu
+
+
+def _noalloc(nd, tape, p, o, loss, grad):
+    import torch
+    lib = nd.load()
+    return lib.ndvm_value_and_grad_noalloc(
+        tape.handle, 0 if p.dtype == torch.float64 else 1, p.shape[0], ctypes.c_void_p(p.data_ptr()),
+        ctypes.c_void_p(o.data_ptr()) if o is not None else None, 0 if o is None else o.numel(),
+        ctypes.c_void_p(loss.data_ptr()), ctypes.c_void_p(grad.data_ptr()),
+        ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+
+
+@pytest.mark.parametrize("make", [lambda: W.logistic(B=3000), lambda: W.random_exprs(2, B=700, n_points=256)[1]],
+                         ids=["workspace-tape", "data-axis-tape"])
+def test_noalloc_matches_regular_entry_point_twice(ndvm, cuda, make):
+    import torch
+    w = make()
+    tape = ndvm.trace_build(w.program, w.frontend)
+    p = torch.tensor(w.params, dtype=torch.float64, device="cuda")
+    o = torch.tensor(w.obs, dtype=torch.float64, device="cuda")
+    ref_loss, ref_grad = ndvm.value_and_grad(tape, p, o)  # also makes the tape resident
+    torch.cuda.synchronize()
+    rl, rg = ref_loss.cpu().numpy(), ref_grad.cpu().numpy()
+    loss, grad = torch.empty_like(ref_loss), torch.empty_like(ref_grad)  # outputs come from the caller
+    for _ in range(2):
+        loss.fill_(float("nan"))
+        grad.fill_(float("nan"))
+        st = _noalloc(ndvm, tape, p, o, loss, grad)
+        assert st == 0, ndvm.load().ndvm_last_error()
+        torch.cuda.synchronize()
+        ok, rep = rel_check(loss.cpu().numpy(), grad.cpu().numpy(), rl, rg, 1e-12)
+        assert ok, rep
+
+
+def test_noalloc_refuses_instead_of_allocating(ndvm, cuda):
+    import torch
+    # a tape whose workspace for one block of lanes exceeds the fixed scratch
+    big = W.kalman_rand8(B=64, T=1000)
+    tape = ndvm.trace_build(big.program)
+    p = torch.tensor(big.params, dtype=torch.float64, device="cuda")
+    o = torch.tensor(big.obs, dtype=torch.float64, device="cuda")
+    loss, grad = torch.empty(64, dtype=torch.float64, device="cuda"), torch.empty_like(p)
+    assert _noalloc(ndvm, tape, p, o, loss, grad) == 1
+    assert b"fixed scratch" in ndvm.load().ndvm_last_error()
+    # a tape never used on this device is not resident: refused, nothing uploaded
+    w = W.logistic(B=8)
+    fresh = ndvm.trace_build(w.program, w.frontend)
+    p2 = torch.tensor(w.params, dtype=torch.float64, device="cuda")
+    o2 = torch.tensor(w.obs, dtype=torch.float64, device="cuda")
+    l2, g2 = torch.empty(8, dtype=torch.float64, device="cuda"), torch.empty_like(p2)
+    assert _noalloc(ndvm, fresh, p2, o2, l2, g2) == 1
+    assert b"not resident" in ndvm.load().ndvm_last_error()
+    np.testing.assert_equal(np.isfinite(p2.cpu().numpy()).all(), True)
