@@ -114,6 +114,19 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def workload_for(args, seed):
+    """(list of Workloads, description) of the configuration being measured."""
+    if args.config == 2:
+        progs = W.random_exprs(n_programs=args.programs, B=B_LANES, n_points=N_POINTS, seed=seed)
+        return progs, WORKLOAD
+    w = W.config(args.config, seed=seed)
+    desc = {1: "exp-decay y = a exp(-b t) + c: 64 lanes x 50 points, MSE",
+            3: "logistic Euler (stack bytecode): 16384 lanes x 1000 steps, 100 obs, MSE",
+            4: "4-state constant-velocity Kalman NLL: 8192 lanes x 200 steps",
+            5: "8-state random stable Kalman NLL: 65536 lanes x 1000 steps"}[args.config]
+    return [w], f"{desc}, {args.dtype} value+grad"
+
+
 def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int):
     """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program."""
     import oracle
@@ -160,6 +173,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
     ap.add_argument("--programs", type=int, default=N_PROGRAMS, help="programs per step (smaller for profiling)")
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5],
+                    help="workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other configurations")
+    ap.add_argument("--dtype", default="f64", choices=["f64", "f32"])
     ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
     ap.add_argument("--cpu-lanes", type=int, default=1024, help="oracle lanes per program for cpu_baseline")
     ap.add_argument("--streams", type=int, default=4, help="CUDA streams the programs are spread over")
@@ -182,12 +198,14 @@ def main():
     nd.load()
 
     # ---- workload: programs traced once on the host; inputs resident in HBM
-    progs = W.random_exprs(n_programs=args.programs, B=B_LANES, n_points=N_POINTS, seed=rank_seed(rank))
+    progs, workload = workload_for(args, rank_seed(rank))
+    tdt = torch.float32 if args.dtype == "f32" else torch.float64
+    npdt = np.float32 if args.dtype == "f32" else np.float64
     t0 = time.perf_counter()
     tapes = [nd.trace_build(w.program, w.frontend) for w in progs]
     trace_s = time.perf_counter() - t0
-    params = [torch.tensor(w.params, dtype=torch.float64, device=dev) for w in progs]
-    obs = [torch.tensor(w.obs, dtype=torch.float64, device=dev) for w in progs]
+    params = [torch.tensor(w.params, dtype=tdt, device=dev) for w in progs]
+    obs = [torch.tensor(w.obs, dtype=tdt, device=dev) for w in progs]
     loss = [torch.empty(w.B, dtype=torch.float64, device=dev) for w in progs]
     grad = [torch.empty_like(p) for p in params]
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
@@ -244,14 +262,14 @@ def main():
     step_ms = [a.elapsed_time(b) for a, b in ev]
     ms = max_over_ranks(float(np.mean(step_ms)), dev)
     clk = clocks.stop()
-    lanes_per_step = args.programs * B_LANES * world
+    lanes_per_step = sum(w.B for w in progs) * world
     value = lanes_per_step / (ms * 1e-3)
 
     # ---- end to end through the host-buffer entry point (pinned host memory)
-    hp = [torch.tensor(w.params, dtype=torch.float64).pin_memory().numpy() for w in progs]
-    ho = [torch.tensor(w.obs, dtype=torch.float64).pin_memory().numpy() for w in progs]
+    hp = [torch.tensor(w.params, dtype=tdt).pin_memory().numpy() for w in progs]
+    ho = [torch.tensor(w.obs, dtype=tdt).pin_memory().numpy() for w in progs]
     h2d = sum(a.nbytes for a in hp) + sum(a.nbytes for a in ho)
-    d2h = sum(w.B * 8 * (1 + w.P) for w in progs)
+    d2h = sum(w.B * np.dtype(npdt).itemsize * (1 + w.P) for w in progs)
 
     def e2e_step():
         for k in range(args.programs):
@@ -286,8 +304,8 @@ def main():
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "programs": args.programs, "lanes_per_program": B_LANES,
+            "vs_baseline": None, "dtype": args.dtype, "data": "synthetic",
+            "config": {"workload": workload, "programs": len(progs), "lanes_per_program": progs[0].B,
                        "points": N_POINTS, "seed": SEED, "l2": "flushed (256 MB write) before every timed step",
                        "parallelism": f"lanes sharded, dp{world}", "streams": args.streams},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},

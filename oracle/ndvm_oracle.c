@@ -31,8 +31,8 @@
  * Readings of points the paper leaves open (all listed in the design doc):
  *   R1  tanh, neg, select, compare, param/obs loads and matrix add/sub/scale are
  *       not in Appendix C: tanh' = 1 - z^2, neg' = -1, select passes the adjoint
- *       to the branch the lane took (section 6, "adjoints gated to the lanes that
- *       took each path"), comparisons carry no gradient.
+ *       to the branch the lane took (section 6: only lanes that took a side send
+ *       adjoints into it), comparisons carry no gradient.
  *   R2  sqrt/log clamp (Appendix C): forward on max(x, 1e-8); zero gradient
  *       unless x > 1e-8 strictly.  abs'(x) = sign(x) with sign(0) = 0.
  *   R3  integer powers (pow with a structural integer exponent n >= 0): forward by
@@ -47,7 +47,7 @@
  *       z = x0 / (x1 * ... * xn) for div, sums and products left to right;
  *       single-argument - and / are negation and reciprocal.
  *   R7  (data-sum N S [BASE] body) sums body over the data axis (section 3.5,
- *       "data" named axis) left to right; (dobs k) inside body reads
+ *       data points as a batch axis) left to right; (dobs k) inside body reads
  *       obs[BASE + d*S + k] for data point d.
  */
 #define _GNU_SOURCE
@@ -1459,7 +1459,7 @@ static Num* run_bytecode(Ctx* cx) {
 }
 
 /* ------------------------------------------------------------------------- */
-/* Lane loop and threading (section 6 "Across cores": one interpreter per     */
+/* Lane loop and threading (section 6, multicore execution: one interpreter per  */
 /* worker, results placed by lane index).                                     */
 /* ------------------------------------------------------------------------- */
 typedef struct {

@@ -6,7 +6,7 @@
 // observations) carry no arithmetic; every other node is one primitive of the
 // Appendix C table (plus tanh, neg, select, compare, matrix add/sub/scale).
 //
-// A data-axis region (section 3.5, the "data" named axis) is a contiguous run of
+// A data-axis region (section 3.5: data points as one of the batch axes) is a contiguous run of
 // body nodes [a, b) followed by a DSUM node that sums the body result over N data
 // points; inside the body, DOBS k reads obs[base + d*stride + k] for point d.
 #pragma once

@@ -87,9 +87,9 @@ def exp_decay(B: int = 64, n_points: int = 50, seed: int = 1234) -> Workload:
 # 2. random expression programs (the paper's typed program generator, section 6)
 # --------------------------------------------------------------------------
 # Grammar: + - * / exp log|x| sin pow-int over x and constants theta_k.
-# Domain guards follow the paper's generator: a division denominator d is wrapped
-# to 1 + d*d, a log argument a to 1 + a*a (inside log|.|), an exp argument a is
-# squashed to a / (1 + a*a).  A program is kept only if every intermediate value
+# Domain guards in the spirit of the paper's generator (section 6): a division by d
+# divides by 1 + d*d instead, a log argument a becomes 1 + a*a (inside log|.|), an exp
+# argument a becomes a / (1 + a*a), bounded by 1/2.  A program is kept only if every intermediate value
 # stays within 1e4 in magnitude at the hidden constants and at sampled lanes.
 
 _BIN = ("+", "-", "*", "/")
