@@ -179,6 +179,8 @@ def main():
     ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
     ap.add_argument("--cpu-lanes", type=int, default=1024, help="oracle lanes per program for cpu_baseline")
     ap.add_argument("--streams", type=int, default=4, help="CUDA streams the programs are spread over")
+    ap.add_argument("--no-graph", dest="graph", action="store_false",
+                    help="launch every step from the host instead of replaying a captured CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:
@@ -219,25 +221,41 @@ def main():
     side = [torch.cuda.Stream(dev) for _ in range(args.streams)]
 
     def step():
+        cur = torch.cuda.current_stream(dev)  # the capture stream while a graph is captured
         if args.streams <= 1:
-            for k in range(args.programs):
-                nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=stream)
+            for k in range(len(tapes)):
+                nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=cur)
             return
         start = torch.cuda.Event()
-        start.record(stream)
+        start.record(cur)
         done = []
         for j, s in enumerate(side):
             s.wait_event(start)
-            for k in range(j, args.programs, args.streams):
+            for k in range(j, len(tapes), args.streams):
                 nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=s)
             e = torch.cuda.Event()
             e.record(s)
             done.append(e)
         for e in done:
-            stream.wait_event(e)
+            cur.wait_event(e)
 
     for _ in range(args.warmup):
         step()
+    torch.cuda.synchronize()
+    # the timed step replays a CUDA graph of one whole step (all programs, all streams):
+    # host launch overhead is paid once at capture, as a deployed calibration loop would
+    per_step_launches = 0
+    graph = None
+    if args.graph:
+        l_cap = nd.launch_count()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            step()
+        per_step_launches = nd.launch_count() - l_cap
+        graph.replay()
+        torch.cuda.synchronize()
+    run_step = graph.replay if graph is not None else step
+
     torch.cuda.synchronize()
     peak_flops = nd.measure_fp64_peak()
 
@@ -254,11 +272,11 @@ def main():
     for i in range(args.steps):
         flush.zero_()
         ev[i][0].record(stream)
-        step()
+        run_step()
         ev[i][1].record(stream)
     torch.cuda.synchronize()
     wall = time.perf_counter() - wall0
-    launches = nd.launch_count() - l0
+    launches = nd.launch_count() - l0 + per_step_launches * args.steps
     step_ms = [a.elapsed_time(b) for a, b in ev]
     ms = max_over_ranks(float(np.mean(step_ms)), dev)
     clk = clocks.stop()
@@ -272,7 +290,7 @@ def main():
     d2h = sum(w.B * np.dtype(npdt).itemsize * (1 + w.P) for w in progs)
 
     def e2e_step():
-        for k in range(args.programs):
+        for k in range(len(tapes)):
             nd.value_and_grad_host(tapes[k], hp[k], ho[k])
 
     e2e_step()
@@ -298,7 +316,7 @@ def main():
         oracle_sample_time(progs[:2], 2, cores)
         n, dt = oracle_sample_time(progs, args.cpu_lanes, cores)
         cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{args.cpu_lanes} lanes of each of the {args.programs} programs ({n} lane evals, {dt:.1f} s)"}
+               "sample": f"{args.cpu_lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals, {dt:.1f} s)"}
 
     if rank == 0:
         line = {
@@ -309,7 +327,7 @@ def main():
                        "points": N_POINTS, "seed": SEED, "l2": "flushed (256 MB write) before every timed step",
                        "parallelism": f"lanes sharded, dp{world}", "streams": args.streams},
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": launches // max(1, args.steps) * args.steps,
+            "gpu_launches": launches, "graph": graph is not None,
             "roofline": roofline,
             "cpu_baseline": cpu,
             "clocks": clk,

@@ -74,7 +74,8 @@ ndvm_status upload_plan(const Tape& t, const Plan& p, DevPlan& d) {
   std::vector<int32_t> args = p.args;
   if (args.empty()) args.push_back(0);
   cudaError_t e;
-  if ((e = cudaMalloc(&d.code, sizeof(DInst) * (p.code.size() ? p.code.size() : 1))) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+  // one spare record: staged copies move 16-byte pieces and may read up to 15 bytes past the end
+  if ((e = cudaMalloc(&d.code, sizeof(DInst) * (p.code.size() + 1))) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
   if ((e = cudaMalloc(&d.args, sizeof(int32_t) * args.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
   if ((e = cudaMalloc(&d.consts_d, sizeof(double) * c.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
   if ((e = cudaMalloc(&d.consts_f, sizeof(float) * cf.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
@@ -125,21 +126,61 @@ int threads_per_lane_override() {
   return v;
 }
 
-// threads per block and threads per lane for a plan
-void launch_shape(const Plan& p, size_t elem, int64_t B, int& tpb, int& log2g) {
-  log2g = 0;
+// Launch shape of a plan: threads per block, threads per lane (1 << log2g), slot-file
+// layout and shared memory per block.
+struct Shape {
+  int tpb = 128, log2g = 0, shared = 0, sstride = 128;
+  int staged = 0, stage_off = 0;
+  size_t smem = 0;
+};
+
+int ilog2(int g) {
+  int l = 0;
+  while ((1 << l) < g) l++;
+  return l;
+}
+
+Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
+  Shape s;
+  const int ov = threads_per_lane_override();
   if (p.has_regions && p.n_save == 0) {
-    // split the data axis over a group of threads when lanes alone cannot fill the GPU
-    const int64_t target = 152LL * 512;
-    int g = threads_per_lane_override();
+    // data-axis tapes: a lane's points split over a thread group, one slot column per thread
+    int g = ov;
     if (!g) {
       g = 1;
-      while (g < 32 && B * g < target) g *= 2;
+      while (g < 32 && B * g < 152LL * 512) g *= 2;
     }
-    while ((1 << log2g) < g) log2g++;
+    s.log2g = ilog2(g);
+    while (s.tpb > 32 && (size_t)p.n_slots * s.tpb * elem > kSmemLimit) s.tpb /= 2;
+    s.sstride = s.tpb;
+  } else if (p.has_matrix) {
+    // matrix tapes: G threads share a lane's slot column and split matrix elements;
+    // G is large enough to give every SMSP two warps and to fit two 128-thread
+    // blocks per SM in shared memory
+    int g = ov > 16 ? 16 : ov;
+    if (!g) {
+      int gf = 1, gs = 1;
+      while (gf < 16 && B * gf < 152LL * 4 * 64) gf *= 2;
+      while (gs < 16 && (size_t)p.n_slots * (128 / gs + 1) * elem > kSmemLimit / 2) gs *= 2;
+      g = gf > gs ? gf : gs;
+    }
+    while (g < 16 && (size_t)p.n_slots * (128 / g + 1) * elem > kSmemLimit) g *= 2;
+    s.log2g = ilog2(g);
+    s.shared = 1;
+    s.sstride = 128 / g + 1;
+  } else {
+    while (s.tpb > 32 && (size_t)p.n_slots * s.tpb * elem > kSmemLimit) s.tpb /= 2;
+    s.sstride = s.tpb;
   }
-  tpb = 128;
-  while (tpb > 32 && (size_t)p.n_slots * tpb * elem > kSmemLimit) tpb /= 2;
+  s.smem = (size_t)p.n_slots * s.sstride * elem;
+  // long loop-free streams are staged through shared memory in double-buffered chunks
+  const size_t stage_bytes = 2 * kStageChunk * sizeof(DInst);
+  if (!p.has_regions && p.code.size() > 2 * (size_t)kStageChunk && s.smem + stage_bytes + 16 <= kSmemLimit) {
+    s.staged = 1;
+    s.stage_off = (int)((s.smem + 15) / 16 * 16);
+    s.smem = s.stage_off + stage_bytes;
+  }
+  return s;
 }
 
 ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
@@ -156,9 +197,9 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   if (n_obs < p.n_obs_min) return fail(NDVM_E_INVALID_ARG, "obs holds " + std::to_string(n_obs) + " values but the program reads " + std::to_string(p.n_obs_min));
   if (p.n_obs_min > 0 && !obs) return fail(NDVM_E_INVALID_ARG, "null obs");
   const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
-  int tpb, log2g;
-  launch_shape(p, elem, B, tpb, log2g);
-  const size_t smem = (size_t)p.n_slots * tpb * elem;
+  const Shape sh = launch_shape(p, elem, B);
+  const int tpb = sh.tpb, log2g = sh.log2g;
+  const size_t smem = sh.smem;
   if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs " + std::to_string(p.n_slots) + " slots per lane, more than shared memory holds");
   const int lanes_per_block = tpb >> log2g;
   int64_t chunk = B;
@@ -190,6 +231,10 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   a.save_ld = chunk;
   a.P = p.n_params;
   a.log2g = log2g;
+  a.shared_lane = sh.shared;
+  a.sstride = sh.sstride;
+  a.staged = sh.staged;
+  a.stage_off = sh.stage_off;
   a.err = dc->err;
   for (int64_t l0 = 0; l0 < B; l0 += chunk) {
     a.lane0 = l0;
@@ -402,9 +447,9 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   if (n_obs < p.n_obs_min) return fail(NDVM_E_INVALID_ARG, "obs holds fewer values than the program reads");
   if (p.n_obs_min > 0 && !obs) return fail(NDVM_E_INVALID_ARG, "null obs");
   const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
-  int tpb, log2g;
-  launch_shape(p, elem, B, tpb, log2g);
-  const size_t smem = (size_t)p.n_slots * tpb * elem;
+  const Shape sh = launch_shape(p, elem, B);
+  const int tpb = sh.tpb, log2g = sh.log2g;
+  const size_t smem = sh.smem;
   if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs more slots per lane than shared memory holds");
   const int lanes_per_block = tpb >> log2g;
   int64_t chunk = B;
@@ -446,6 +491,10 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   a.save_ld = chunk;
   a.P = p.n_params;
   a.log2g = log2g;
+  a.shared_lane = sh.shared;
+  a.sstride = sh.sstride;
+  a.staged = sh.staged;
+  a.stage_off = sh.stage_off;
   a.err = dc->err;
   for (int64_t l0 = 0; l0 < B; l0 += chunk) {
     a.lane0 = l0;

@@ -13,6 +13,7 @@
 
 #include <algorithm>
 #include <climits>
+#include <cstdlib>
 #include <cstring>
 #include <set>
 
@@ -23,6 +24,12 @@ namespace ndvm {
 namespace {
 
 [[noreturn]] void unsupported(const std::string& m) { throw BuildError{NDVM_E_UNSUPPORTED, m}; }
+
+// NDVM_PREFETCH=0 disables the reverse sweep's workspace prefetch (a tuning knob).
+bool prefetch_enabled() {
+  const char* e = std::getenv("NDVM_PREFETCH");
+  return !(e && e[0] == '0');
+}
 
 struct PRef {
   uint32_t kind = RK_SLOT;
@@ -99,7 +106,9 @@ class Planner {
   std::pair<PRef, bool> target(int x);
   void emit_reverse(int v);
   void allocate();
+  void prefetch_workspace();
   int32_t encode(const PArg& a) const;
+  int rev_begin_ = -1;  // first instruction of the reverse sweep
 };
 
 std::vector<int> Planner::inputs(int v) const {
@@ -521,6 +530,79 @@ void Planner::emit_region(int v) {
   emit(gr);
 }
 
+// Software pipeline for the reverse sweep of a spill tape: the scalar workspace
+// values that reverse instruction j reads are fetched (asynchronous copies into a
+// ring of slots) kFetchDepth instructions earlier, so the HBM latency overlaps the
+// preceding instructions instead of stalling each one.
+void Planner::prefetch_workspace() {
+  if (rev_begin_ < 0) return;
+  auto scalar_fields = [](uint8_t op, int* fl) -> int {
+    int n = 0;
+    switch (op) {
+      case B_MUL: fl[n++] = 3; fl[n++] = 4; break;
+      case B_DIV: fl[n++] = 4; fl[n++] = 5; break;
+      case B_POW: fl[n++] = 3; fl[n++] = 4; fl[n++] = 5; break;
+      case B_EXP: case B_TANH: fl[n++] = 5; break;
+      case B_LOG: case B_ABS: case B_POWI: case B_SELECT: case B_MSCALE: fl[n++] = 3; break;
+      case B_SQRT: fl[n++] = 3; fl[n++] = 5; break;
+      case B_SIN: case B_COS: fl[n++] = 6; break;
+      case B_DET: fl[n++] = 5; break;
+      default: break;
+    }
+    return n;
+  };
+  const int nsteps = (int)code_.size() - rev_begin_;
+  std::vector<std::vector<int>> reads(nsteps);
+  size_t total = 0;
+  for (int j = 0; j < nsteps; j++) {
+    const PInst& p = code_[rev_begin_ + j];
+    int fl[4];
+    int n = scalar_fields(p.d.op, fl);
+    for (int k = 0; k < n; k++)
+      if (p.f[fl[k]].isref && p.f[fl[k]].r.kind == RK_SAVE) reads[j].push_back(fl[k]);
+    total += reads[j].size();
+  }
+  if (total == 0) return;
+  // ring capacity: the most reads in flight over any kFetchDepth + 1 consecutive steps
+  int ring = 0, window = 0;
+  for (int j = 0; j < nsteps; j++) {
+    window += (int)reads[j].size();
+    if (j > kFetchDepth) window -= (int)reads[j - kFetchDepth - 1].size();
+    ring = std::max(ring, window);
+  }
+  ring += 1;
+  const int ring_vr = new_vr(ring);
+  // assign ring entries in consumption order and rewrite the consumers
+  std::vector<std::vector<std::pair<PArg, PArg>>> fetch(nsteps);
+  int counter = 0;
+  for (int j = 0; j < nsteps; j++) {
+    PInst& p = code_[rev_begin_ + j];
+    for (int fld : reads[j]) {
+      PArg slot = R(slotref(ring_vr, counter % ring));
+      counter++;
+      fetch[j].push_back({p.f[fld], slot});
+      p.f[fld] = slot;
+    }
+  }
+  auto fetch_inst = [&](int j, bool wait) {
+    PInst f;
+    f.d.op = D_FETCH;
+    f.d.flags = wait ? 1 : 0;
+    f.f[1] = I((int32_t)args_.size());
+    f.f[2] = I(j < nsteps ? (int32_t)fetch[j].size() : 0);
+    if (j < nsteps)
+      for (auto& pr : fetch[j]) { args_.push_back(pr.first); args_.push_back(pr.second); }
+    return f;
+  };
+  std::vector<PInst> out(code_.begin(), code_.begin() + rev_begin_);
+  for (int j = 0; j < kFetchDepth; j++) out.push_back(fetch_inst(j, false));  // prologue
+  for (int j = 0; j < nsteps; j++) {
+    out.push_back(fetch_inst(j + kFetchDepth, true));
+    out.push_back(code_[rev_begin_ + j]);
+  }
+  code_.swap(out);
+}
+
 int32_t Planner::encode(const PArg& a) const {
   if (!a.isref) return a.v;
   if (a.r.kind == RK_SLOT) {
@@ -548,6 +630,7 @@ void Planner::allocate() {
       case D_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 1; break;
       case B_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 2; break;
       case B_DSUM: off = p.f[1].v; cnt = p.f[2].v; stride = 3; break;
+      case D_FETCH: off = p.f[1].v; cnt = p.f[2].v; stride = 2; break;
       default: break;
     }
     if (off >= 0)
@@ -605,6 +688,7 @@ Plan Planner::build() {
   }
   PInst ls; ls.d.op = D_LOSS; ls.f[0] = R(ref(T.loss));
   emit(ls);
+  rev_begin_ = (int)code_.size();
   if (grad_) {
     if (active_[T.loss]) {
       if (is_leaf(T.loss)) {
@@ -630,6 +714,7 @@ Plan Planner::build() {
       emit(g);
     }
   }
+  if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
   allocate();
   pl.n_slots = n_slots_;
   pl.n_save = S_;
@@ -642,6 +727,10 @@ Plan Planner::build() {
     pl.code.push_back(d);
   }
   for (const PArg& a : args_) pl.args.push_back(encode(a));
+  for (const DInst& d : pl.code)
+    if (d.op == D_MATMUL || d.op == D_MADD || d.op == D_MSUB || d.op == D_MSCALE || d.op == D_INV ||
+        ((d.op == D_DET || d.op == D_LOGDET) && d.r > 1) || (d.op == D_GATHER && d.f[2] > 1))
+      pl.has_matrix = true;
   pl.extra_consts = extra_consts_;
   pl.work_fwd = work_fwd_;
   pl.work_rev = work_rev_;
@@ -775,6 +864,13 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
             ok = ok && ref_ok(p.args[f[1] + 3 * e], 1, true) && p.args[f[1] + 3 * e] != -1 && ref_ok(p.args[f[1] + 3 * e + 2], 1, true);
         break;
       case B_GRAD: ok = ref_ok(f[0], 1, true) && f[1] >= 0 && f[1] < p.n_params; break;
+      case D_FETCH:
+        ok = args_ok(f[1], f[2], 2);
+        if (ok)
+          for (int e = 0; e < f[2]; e++)
+            ok = ok && ref_kind(p.args[f[1] + 2 * e]) == RK_SAVE && ref_ok(p.args[f[1] + 2 * e], 1, false) &&
+                 ref_ok(p.args[f[1] + 2 * e + 1], 1, true);
+        break;
       default: why = "bad opcode"; return false;
     }
     if (!ok) { why = "operand out of range at instruction " + std::to_string(pc) + " (op " + std::to_string(d.op) + ")"; return false; }

@@ -71,8 +71,16 @@ enum DOp : uint8_t {
   B_TRACE,          // f1 gA; n = r
   B_DSUM,           // f1 args offset, f2 count (args: triples target slot, first flag, partial slot)
   B_GRAD,           // grad[lane, f1] = slot f0 (or 0 if f0 < 0)
+  // ---- workspace prefetch (reverse sweep of long tapes) ----
+  D_FETCH,          // f1 args offset, f2 count (args: pairs workspace ref, slot ref): asynchronous
+                    // copies into slots, committed as one group; flags bit0: then wait until at
+                    // most kFetchDepth groups are pending
   D_NOPS
 };
+
+// Reverse instructions read their workspace values from slots filled this many
+// instructions ahead.
+constexpr int kFetchDepth = 8;
 
 struct DInst {
   uint8_t op = 0, r = 1, c = 1, k = 1;
@@ -85,6 +93,7 @@ struct Plan {
   bool grad = false;          // has a reverse sweep
   bool spill = false;         // reverse reads primals from the HBM workspace
   bool has_regions = false;   // contains data-axis loops
+  bool has_matrix = false;    // contains instructions over matrices
   int32_t n_slots = 0;        // per-lane slot file size (elements)
   int64_t n_save = 0;         // per-lane workspace elements
   int32_t n_params = 0;

@@ -37,10 +37,11 @@ struct Opnd {
   __device__ __forceinline__ T operator[](int e) const { return p[(int64_t)e * s]; }
 };
 
-template <typename T>
+template <typename T, bool SHARED>
 struct Lane {
-  T* slots;
-  int tpb, tid;
+  T* sbase;           // this thread's slot column: element s of the slot file is sbase[s * ss]
+  int ss;             // slot row stride in elements
+  int eg, emask;      // SHARED: this thread writes the elements e with (e & emask) == eg
   const T* consts;
   const T* obs;
   const T* params;
@@ -51,8 +52,8 @@ struct Lane {
   __device__ __forceinline__ Opnd<T> rd(int32_t ref) const {
     const uint32_t kind = ((uint32_t)ref >> 28) & 7u;
     const int32_t idx = ref & kRefIndexMask;
+    if (kind == RK_SLOT) return {sbase + idx * ss, ss};
     switch (kind) {
-      case RK_SLOT: return {slots + (int64_t)idx * tpb + tid, tpb};
       case RK_CONST: return {consts + idx, 1};
       case RK_OBS: return {obs + idx, 1};
       case RK_DOBS: return {obs + dbase + idx, 1};
@@ -60,18 +61,27 @@ struct Lane {
       default: return {params + lane * P + idx, 1};
     }
   }
-  __device__ __forceinline__ T ld(int32_t ref) const { return rd(ref)[0]; }
+  __device__ __forceinline__ T ld(int32_t ref) const {
+    if (((uint32_t)ref >> 28) == RK_SLOT) return sbase[ref * ss];
+    return rd(ref)[0];
+  }
+  __device__ __forceinline__ bool own(int e) const { return SHARED ? ((e & emask) == eg) : true; }
+  __device__ __forceinline__ int step() const { return SHARED ? emask + 1 : 1; }
+  __device__ __forceinline__ int first() const { return SHARED ? eg : 0; }
   // slot references only
-  __device__ __forceinline__ T* wp(int32_t ref) const { return slots + (int64_t)(ref & kRefIndexMask) * tpb + tid; }
-  __device__ __forceinline__ void st(int32_t ref, int e, T v) const { wp(ref)[(int64_t)e * tpb] = v; }
-  __device__ __forceinline__ T sl(int32_t ref, int e) const { return wp(ref)[(int64_t)e * tpb]; }
-  // adjoint update: first contribution stores, later ones accumulate
+  __device__ __forceinline__ T* wp(int32_t ref) const { return sbase + (ref & kRefIndexMask) * ss; }
+  __device__ __forceinline__ T sl(int32_t ref, int e) const { return wp(ref)[e * ss]; }
+  __device__ __forceinline__ void st(int32_t ref, int e, T v) const {
+    if (own(e)) wp(ref)[e * ss] = v;
+  }
+  // adjoint update: the first contribution stores, later ones accumulate
   __device__ __forceinline__ void upd(int32_t ref, int e, T v, bool first) const {
-    T* q = wp(ref) + (int64_t)e * tpb;
+    if (!own(e)) return;
+    T* q = wp(ref) + e * ss;
     *q = first ? v : *q + v;
   }
   __device__ __forceinline__ void save_out(int32_t sidx, int e, T v) const {
-    if (sidx >= 0) save[(int64_t)(sidx + e) * save_ld + col] = v;
+    if (sidx >= 0 && own(e)) save[(int64_t)(sidx + e) * save_ld + col] = v;
   }
 };
 
@@ -168,33 +178,50 @@ __device__ T det_inv(const Opnd<T>& A, int n, T* inv /* n*n or nullptr */) {
   return d;
 }
 
-template <typename T>
-__device__ __forceinline__ bool all_zero(const Lane<T>& L, int32_t gz, int w) {
+template <typename LaneT>
+__device__ __forceinline__ bool all_zero(const LaneT& L, int32_t gz, int w) {
   for (int e = 0; e < w; e++)
     if (!is_zero(L.sl(gz, e))) return false;
   return true;
 }
-template <typename T>
-__device__ __forceinline__ void zero_if_first(const Lane<T>& L, int32_t ref, int w, bool first) {
+template <typename LaneT>
+__device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w, bool first) {
   if (first && ref != -1)
-    for (int e = 0; e < w; e++) L.st(ref, e, (T)0);
+    for (int e = L.first(); e < w; e += L.step()) L.wp(ref)[e * L.ss] = 0;
 }
 
-template <typename T>
+// Two layouts of the slot file.  Per-thread (shared_lane = 0): every thread owns a
+// lane -- or, for data-axis tapes, a share of a lane's data points -- and its own
+// column of slots.  Per-lane (shared_lane = 1): the G threads of a lane share one
+// column; each matrix instruction's output elements are split over them (element e
+// belongs to thread e mod G), scalar instructions are computed by all G and written
+// by the owner of element 0, and a warp barrier after every instruction publishes
+// the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
+// cost while G times more warps cover the lanes.
+template <typename T, bool SHARED, bool STAGED>
 __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
   const int G = 1 << a.log2g;
-  const int64_t lane_raw = a.lane0 + (int64_t)blockIdx.x * (tpb >> a.log2g) + (tid >> a.log2g);
+  const int lane_in_block = tid >> a.log2g;
+  const int64_t lane_raw = a.lane0 + (int64_t)blockIdx.x * (tpb >> a.log2g) + lane_in_block;
   const int grank = tid & (G - 1);
   const bool live = lane_raw < a.lane_end;
-  if (G == 1 && !live) return;
+  if (G == 1 && !live && !STAGED) return;  // staged blocks keep every thread for the block barriers
 
-  Lane<T> L;
-  L.slots = reinterpret_cast<T*>(smem_raw);
-  L.tpb = tpb;
-  L.tid = tid;
+  Lane<T, SHARED> L;
+  if (SHARED) {
+    L.ss = a.sstride;
+    L.sbase = reinterpret_cast<T*>(smem_raw) + lane_in_block;
+    L.eg = grank;
+    L.emask = G - 1;
+  } else {
+    L.ss = tpb;
+    L.sbase = reinterpret_cast<T*>(smem_raw) + tid;
+    L.eg = 0;
+    L.emask = 0;
+  }
   L.consts = static_cast<const T*>(a.consts);
   L.obs = static_cast<const T*>(a.obs);
   L.params = static_cast<const T*>(a.params);
@@ -207,14 +234,55 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
   T* loss = static_cast<T*>(a.loss);
   T* grad = static_cast<T*>(a.grad);
   const bool writer = live && grank == 0;
+  const bool sync_each = SHARED && G > 1;
+  const int es = L.step();
 
   int64_t d = 0, dN = 0, dstride = 0, dbase0 = 0;
   int loop_pc = -1;
   const DInst* __restrict__ code = a.code;
   const int32_t* __restrict__ args = a.args;
 
+  // Staged instruction stream: chunk k of kStageChunk instructions sits in buffer
+  // k % 2; the copy of chunk k + 1 is in flight while chunk k executes.  Every
+  // thread of the block runs the same instruction sequence (staged plans have no
+  // data-axis loops), so the block barrier at each chunk boundary is uniform.
+  DInst* stage = reinterpret_cast<DInst*>(smem_raw + a.stage_off);
+  auto stage_copy = [&](int chunk) {
+    const int first = chunk * kStageChunk;
+    if (first >= a.n_code) return;
+    const int n = min(kStageChunk, a.n_code - first);
+    const char* src = reinterpret_cast<const char*>(code + first);
+    char* dst = reinterpret_cast<char*>(stage + (chunk & 1) * kStageChunk);
+    const int pieces = (n * (int)sizeof(DInst) + 15) / 16;  // the device copy is padded to 16 bytes
+    for (int i = tid; i < pieces; i += tpb) {
+      const unsigned d = (unsigned)__cvta_generic_to_shared(dst + 16 * i);
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(d), "l"(src + 16 * i) : "memory");
+    }
+  };
+  if (STAGED) {
+    stage_copy(0);
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+    stage_copy(1);
+    asm volatile("cp.async.commit_group;\n" ::: "memory");
+    asm volatile("cp.async.wait_group 1;\n" ::: "memory");
+    __syncthreads();
+  }
+  // non-staged streams: the record of the next instruction is loaded before the
+  // current one executes, so its latency overlaps the current instruction
+  DInst nxt;
+  if (!STAGED && a.n_code > 0) nxt = code[0];
   for (int pc = 0; pc < a.n_code; pc++) {
-    const DInst in = code[pc];
+    if (STAGED && pc > 0 && (pc % kStageChunk) == 0) {
+      const int k = pc / kStageChunk;
+      __syncthreads();  // every warp has left chunk k - 1: its buffer is free
+      stage_copy(k + 1);
+      asm volatile("cp.async.commit_group;\n" ::: "memory");
+      asm volatile("cp.async.wait_group 1;\n" ::: "memory");  // chunk k has landed
+      __syncthreads();
+    }
+    const DInst in = STAGED ? stage[((pc / kStageChunk) & 1) * kStageChunk + pc % kStageChunk] : nxt;
+    if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
+
     const int32_t* f = in.f;
     const int w = in.r * in.c;
     switch (in.op) {
@@ -244,7 +312,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       case D_SIN: case D_COS: {
         T x = L.ld(f[1]);
-        T s, c;
+        T s = 0, c = 0;
         if (f[4] != -1 || f[5] >= 0) {
           sincos(x, &s, &c);
           T aux = in.op == D_SIN ? c : s;
@@ -283,7 +351,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       case D_GATHER: {
         const int32_t* g = args + f[1];
-        for (int e = 0; e < f[2]; e++) {
+        for (int e = L.first(); e < f[2]; e += es) {
           T v = L.ld(g[e]);
           L.st(f[0], e, v);
           L.save_out(f[3], e, v);
@@ -292,7 +360,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       case D_MADD: case D_MSUB: {
         Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
-        for (int e = 0; e < w; e++) {
+        for (int e = L.first(); e < w; e += es) {
           T z = in.op == D_MADD ? A[e] + Bm[e] : A[e] - Bm[e];
           L.st(f[0], e, z);
           L.save_out(f[3], e, z);
@@ -302,7 +370,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case D_MSCALE: {
         T s = L.ld(f[1]);
         Opnd<T> A = L.rd(f[2]);
-        for (int e = 0; e < w; e++) {
+        for (int e = L.first(); e < w; e += es) {
           T z = s * A[e];
           L.st(f[0], e, z);
           L.save_out(f[3], e, z);
@@ -311,21 +379,21 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       case D_MATMUL: {
         Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
-        const int r = in.r, c = in.c, kk = in.k;
-        for (int i = 0; i < r; i++)
-          for (int j = 0; j < c; j++) {
-            T s = A[i * kk] * Bm[j];
-            for (int q = 1; q < kk; q++) s = fma(A[i * kk + q], Bm[q * c + j], s);
-            L.st(f[0], i * c + j, s);
-            L.save_out(f[3], i * c + j, s);
-          }
+        const int c = in.c, kk = in.k;
+        for (int e = L.first(); e < w; e += es) {
+          const int i = e / c, j = e - i * c;
+          T s = A[i * kk] * Bm[j];
+          for (int q = 1; q < kk; q++) s = fma(A[i * kk + q], Bm[q * c + j], s);
+          L.st(f[0], e, s);
+          L.save_out(f[3], e, s);
+        }
         break;
       }
       case D_INV: {
         const int n = in.r;
         T inv[64];
         det_inv(L.rd(f[1]), n, inv);
-        for (int e = 0; e < n * n; e++) {
+        for (int e = L.first(); e < n * n; e += es) {
           L.st(f[0], e, inv[e]);
           L.save_out(f[3], e, inv[e]);
         }
@@ -340,7 +408,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
         if (aux)
-          for (int e = 0; e < n * n; e++) {
+          for (int e = L.first(); e < n * n; e += es) {
             if (f[4] != -1) L.st(f[4], e, inv[e]);
             L.save_out(f[5], e, inv[e]);
           }
@@ -356,18 +424,26 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       }
       // ------------------------------------------------------------ data axis
       case D_ZERO:
-        for (int e = 0; e < f[1]; e++) L.st(f[0], e, (T)0);
+        for (int e = L.first(); e < f[1]; e += es) L.st(f[0], e, (T)0);
         break;
       case D_LOOP:
         dN = f[0]; dstride = f[1]; dbase0 = f[2];
         d = grank;
         loop_pc = pc;
-        if (d >= dN) { pc = f[3]; break; }  // resumes after the loop end
+        if (d >= dN) {  // no point for this thread: resume after the loop end
+          pc = f[3];
+          if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
+          break;
+        }
         L.dbase = dbase0 + d * dstride;
         break;
       case D_ENDLOOP:
         d += G;
-        if (d < dN) { L.dbase = dbase0 + d * dstride; pc = loop_pc; }
+        if (d < dN) {
+          L.dbase = dbase0 + d * dstride;
+          pc = loop_pc;
+          if (!STAGED) nxt = code[pc + 1];
+        }
         break;
       case D_ACC: L.st(f[0], 0, L.sl(f[0], 0) + L.ld(f[1])); break;
       case D_SEED: L.st(f[0], 0, (T)1); break;
@@ -450,6 +526,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         break;
       }
       case B_GATHER: {
+        // every target is a scalar (element 0 of its own value)
         const int32_t* g = args + f[1];
         const bool z = all_zero(L, f[0], f[2]);
         for (int e = 0; e < f[2]; e++) {
@@ -467,13 +544,14 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         zero_if_first(L, f[1], f[4], first);
         if (all_zero(L, f[0], f[2])) break;
         const int32_t* m = args + f[3];
-        for (int e = 0; e < f[2]; e++) L.st(f[1], m[e], L.sl(f[1], m[e]) + L.sl(f[0], e));
+        for (int e = 0; e < f[2]; e++)
+          if (L.own(m[e])) L.st(f[1], m[e], L.sl(f[1], m[e]) + L.sl(f[0], e));
         break;
       }
       case B_MADD: case B_MSUB: {
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], w, fa); zero_if_first(L, f[2], w, fb); break; }
-        for (int e = 0; e < w; e++) {
+        for (int e = L.first(); e < w; e += es) {
           T g = L.sl(f[0], e);
           if (f[1] != -1) L.upd(f[1], e, g, fa);
           if (f[2] != -1) L.upd(f[2], e, in.op == B_MADD ? g : -g, fb);
@@ -491,7 +569,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         }
         if (f[2] != -1) {
           T s = L.ld(f[3]);
-          for (int e = 0; e < w; e++) L.upd(f[2], e, s * L.sl(f[0], e), fb);
+          for (int e = L.first(); e < w; e += es) L.upd(f[2], e, s * L.sl(f[0], e), fb);
         }
         break;
       }
@@ -499,24 +577,24 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         const int r = in.r, c = in.c, kk = in.k;
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], r * kk, fa); zero_if_first(L, f[2], kk * c, fb); break; }
-        Opnd<T> G_ = {L.wp(f[0]), L.tpb};
+        Opnd<T> G_ = {L.wp(f[0]), L.ss};
         if (f[1] != -1) {  // gA (r x k) += gZ (r x c) * B^T (B is k x c)
           Opnd<T> Bm = L.rd(f[4]);
-          for (int i = 0; i < r; i++)
-            for (int q = 0; q < kk; q++) {
-              T s = G_[i * c] * Bm[q * c];
-              for (int j = 1; j < c; j++) s = fma(G_[i * c + j], Bm[q * c + j], s);
-              L.upd(f[1], i * kk + q, s, fa);
-            }
+          for (int e = L.first(); e < r * kk; e += es) {
+            const int i = e / kk, q = e - i * kk;
+            T s = G_[i * c] * Bm[q * c];
+            for (int j = 1; j < c; j++) s = fma(G_[i * c + j], Bm[q * c + j], s);
+            L.upd(f[1], e, s, fa);
+          }
         }
         if (f[2] != -1) {  // gB (k x c) += A^T (A is r x k) * gZ
           Opnd<T> A = L.rd(f[3]);
-          for (int q = 0; q < kk; q++)
-            for (int j = 0; j < c; j++) {
-              T s = A[q] * G_[j];
-              for (int i = 1; i < r; i++) s = fma(A[i * kk + q], G_[i * c + j], s);
-              L.upd(f[2], q * c + j, s, fb);
-            }
+          for (int e = L.first(); e < kk * c; e += es) {
+            const int q = e / c, j = e - q * c;
+            T s = A[q] * G_[j];
+            for (int i = 1; i < r; i++) s = fma(A[i * kk + q], G_[i * c + j], s);
+            L.upd(f[2], e, s, fb);
+          }
         }
         break;
       }
@@ -526,7 +604,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         if (f[1] == -1) break;
         if (all_zero(L, f[0], n * n)) { zero_if_first(L, f[1], n * n, fa); break; }
         Opnd<T> Bv = L.rd(f[5]);
-        Opnd<T> G_ = {L.wp(f[0]), L.tpb};
+        Opnd<T> G_ = {L.wp(f[0]), L.ss};
         T m[64];  // M = gZ B^T
         for (int p = 0; p < n; p++)
           for (int j = 0; j < n; j++) {
@@ -534,12 +612,12 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
             for (int q = 1; q < n; q++) s = fma(G_[p * n + q], Bv[j * n + q], s);
             m[p * n + j] = s;
           }
-        for (int i = 0; i < n; i++)  // gA -= B^T M
-          for (int j = 0; j < n; j++) {
-            T s = Bv[i] * m[j];
-            for (int p = 1; p < n; p++) s = fma(Bv[p * n + i], m[p * n + j], s);
-            L.upd(f[1], i * n + j, -s, fa);
-          }
+        for (int e = L.first(); e < n * n; e += es) {  // gA -= B^T M
+          const int i = e / n, j = e - i * n;
+          T s = Bv[i] * m[j];
+          for (int p = 1; p < n; p++) s = fma(Bv[p * n + i], m[p * n + j], s);
+          L.upd(f[1], e, -s, fa);
+        }
         break;
       }
       case B_DET: case B_LOGDET: {
@@ -550,8 +628,10 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         if (is_zero(g)) { zero_if_first(L, f[1], n * n, fa); break; }
         T fac = in.op == B_DET ? g * L.ld(f[5]) : g;
         Opnd<T> Iv = L.rd(f[6]);
-        for (int i = 0; i < n; i++)
-          for (int j = 0; j < n; j++) L.upd(f[1], i * n + j, fac * Iv[j * n + i], fa);
+        for (int e = L.first(); e < n * n; e += es) {
+          const int i = e / n, j = e - i * n;
+          L.upd(f[1], e, fac * Iv[j * n + i], fa);
+        }
         break;
       }
       case B_TRACE: {
@@ -561,7 +641,8 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         T g = L.sl(f[0], 0);
         zero_if_first(L, f[1], n * n, fa);
         if (is_zero(g)) break;
-        for (int i = 0; i < n; i++) L.st(f[1], i * n + i, L.sl(f[1], i * n + i) + g);
+        for (int i = 0; i < n; i++)
+          if (L.own(i * n + i)) L.st(f[1], i * n + i, L.sl(f[1], i * n + i) + g);
         break;
       }
       case B_DSUM: {
@@ -578,27 +659,53 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       case B_GRAD:
         if (writer) grad[L.lane * L.P + f[1]] = f[0] == -1 ? (T)0 : L.sl(f[0], 0);
         break;
+      case D_FETCH: {
+        // asynchronous copies of workspace values into slots (the owner of element 0
+        // copies; the warp barrier after the wait publishes them to the group)
+        const int32_t* q = args + f[1];
+        if (L.own(0))
+          for (int e = 0; e < f[2]; e++) {
+            const T* src = L.rd(q[2 * e]).p;
+            const unsigned dst = (unsigned)__cvta_generic_to_shared(L.wp(q[2 * e + 1]));
+            if (sizeof(T) == 8)
+              asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(src) : "memory");
+            else
+              asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
+          }
+        asm volatile("cp.async.commit_group;\n" ::: "memory");
+        if (in.flags & 1) asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchDepth) : "memory");
+        break;
+      }
       default:
         if (a.err) atomicExch(a.err, 1);
         return;
     }
+    if (sync_each) __syncwarp();
   }
 }
 
-template <typename T>
-cudaError_t launch_t(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
+template <typename T, bool SHARED, bool STAGED>
+cudaError_t launch_v(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
   static int configured_dev = -1;
   static size_t configured_smem = 0;
   int dev = 0;
   cudaGetDevice(&dev);
   if (configured_dev != dev || smem > configured_smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_replay<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_replay<T, SHARED, STAGED>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     configured_dev = dev;
     configured_smem = smem;
   }
-  k_replay<T><<<blocks, tpb, smem, s>>>(a);
+  k_replay<T, SHARED, STAGED><<<blocks, tpb, smem, s>>>(a);
   return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_t(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  if (a.shared_lane)
+    return a.staged ? launch_v<T, true, true>(a, blocks, tpb, smem, s) : launch_v<T, true, false>(a, blocks, tpb, smem, s);
+  return a.staged ? launch_v<T, false, true>(a, blocks, tpb, smem, s) : launch_v<T, false, false>(a, blocks, tpb, smem, s);
 }
 
 }  // namespace

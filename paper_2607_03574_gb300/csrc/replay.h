@@ -23,10 +23,17 @@ struct ReplayArgs {
   int64_t save_ld;       // workspace column count (lanes per chunk)
   int P;
   int log2g;             // threads per lane = 1 << log2g
+  int shared_lane;       // 1: the lane's threads share one slot column and split matrix elements
+  int sstride;           // slot row stride in elements (threads per block, or lanes per block + pad)
   int* err;              // device flag set on an invalid instruction
+  int staged;            // 1: the instruction stream is staged through shared memory in chunks
+  int stage_off;         // byte offset of the two chunk buffers in dynamic shared memory
 };
 
 cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
+
+// Instructions per staged chunk (two chunk buffers of 5 KB sit after the slot file).
+constexpr int kStageChunk = 128;
 
 // Size of the fixed scratch array of the no-allocation entry point (32 MiB).
 constexpr size_t kNoAllocScratchBytes = size_t(32) << 20;

@@ -52,9 +52,10 @@ def test_noalloc_matches_regular_entry_point_twice(ndvm, cuda, make):
 
 def test_noalloc_refuses_instead_of_allocating(ndvm, cuda):
     import torch
-    # a tape whose workspace for one block of lanes exceeds the fixed scratch
-    big = W.kalman_rand8(B=64, T=1000)
-    tape = ndvm.trace_build(big.program)
+    # a tape whose workspace for one block of lanes exceeds the fixed scratch:
+    # 20,000 Euler steps keep about 82,000 values per lane (84 MB per 128-lane block)
+    big = W.logistic(B=64, n_obs=2000)
+    tape = ndvm.trace_build(big.program, big.frontend)
     p = torch.tensor(big.params, dtype=torch.float64, device="cuda")
     o = torch.tensor(big.obs, dtype=torch.float64, device="cuda")
     loss, grad = torch.empty(64, dtype=torch.float64, device="cuda"), torch.empty_like(p)
