@@ -82,12 +82,14 @@ enum DOp : uint8_t {
 // instructions ahead.
 constexpr int kFetchDepth = 8;
 
-struct DInst {
+// 48 bytes, 16-byte aligned: the kernel fetches a record with three 128-bit loads.
+struct alignas(16) DInst {
   uint8_t op = 0, r = 1, c = 1, k = 1;
   uint8_t flags = 0, pad0 = 0, pad1 = 0, pad2 = 0;
   int32_t f[8] = {-1, -1, -1, -1, -1, -1, -1, -1};
+  int32_t pad3 = 0, pad4 = 0;
 };
-static_assert(sizeof(DInst) == 40, "DInst layout");
+static_assert(sizeof(DInst) == 48, "DInst layout");
 
 struct Plan {
   bool grad = false;          // has a reverse sweep

@@ -287,29 +287,36 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
     const int w = in.r * in.c;
     switch (in.op) {
       // ------------------------------------------------------------ forward
-      case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: {
-        T x = L.ld(f[1]), y = L.ld(f[2]), z;
-        if (in.op == D_ADD) z = x + y;
-        else if (in.op == D_SUB) z = x - y;
-        else if (in.op == D_MUL) z = x * y;
-        else if (in.op == D_DIV) z = x / y;
-        else z = pow(x, y);
-        L.st(f[0], 0, z);
-        L.save_out(f[3], 0, z);
-        break;
-      }
-      case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: {
-        T x = L.ld(f[1]), z;
-        if (in.op == D_NEG) z = -x;
-        else if (in.op == D_EXP) z = fast_exp(x);
-        else if (in.op == D_LOG) z = fast_log(gt_eps(x) ? x : clamp_eps<T>());
-        else if (in.op == D_TANH) z = tanh(x);
-        else if (in.op == D_SQRT) z = sqrt(gt_eps(x) ? x : clamp_eps<T>());
-        else z = fabs(x);
-        L.st(f[0], 0, z);
-        L.save_out(f[3], 0, z);
-        break;
-      }
+      // one case per opcode: the switch's jump is the only dispatch branch
+#define NDVM_FWD1(OPC, EXPR)                 \
+  case OPC: {                                \
+    const T x = L.ld(f[1]);                  \
+    const T z = (EXPR);                      \
+    L.st(f[0], 0, z);                        \
+    L.save_out(f[3], 0, z);                  \
+    break;                                   \
+  }
+#define NDVM_FWD2(OPC, EXPR)                 \
+  case OPC: {                                \
+    const T x = L.ld(f[1]), y = L.ld(f[2]);  \
+    const T z = (EXPR);                      \
+    L.st(f[0], 0, z);                        \
+    L.save_out(f[3], 0, z);                  \
+    break;                                   \
+  }
+      NDVM_FWD2(D_ADD, x + y)
+      NDVM_FWD2(D_SUB, x - y)
+      NDVM_FWD2(D_MUL, x * y)
+      NDVM_FWD2(D_DIV, x / y)
+      NDVM_FWD2(D_POW, pow(x, y))
+      NDVM_FWD1(D_NEG, -x)
+      NDVM_FWD1(D_EXP, fast_exp(x))
+      NDVM_FWD1(D_LOG, fast_log(gt_eps(x) ? x : clamp_eps<T>()))
+      NDVM_FWD1(D_TANH, tanh(x))
+      NDVM_FWD1(D_SQRT, sqrt(gt_eps(x) ? x : clamp_eps<T>()))
+      NDVM_FWD1(D_ABS, fabs(x))
+#undef NDVM_FWD1
+#undef NDVM_FWD2
       case D_SIN: case D_COS: {
         T x = L.ld(f[1]);
         T s = 0, c = 0;
@@ -461,12 +468,19 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         if (writer) loss[L.lane] = L.ld(f[0]);
         break;
       // ------------------------------------------------------------ reverse
-      case B_ADD: case B_SUB: case B_NEG: {
-        T g = L.sl(f[0], 0);
-        bool fa = in.flags & 1, fb = in.flags & 2;
-        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); if (in.op != B_NEG) zero_if_first(L, f[2], 1, fb); break; }
-        if (f[1] != -1) L.upd(f[1], 0, in.op == B_NEG ? -g : g, fa);
-        if (in.op != B_NEG && f[2] != -1) L.upd(f[2], 0, in.op == B_ADD ? g : -g, fb);
+      case B_ADD: case B_SUB: {
+        const T g = L.sl(f[0], 0);
+        const bool fa = in.flags & 1, fb = in.flags & 2;
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
+        if (f[1] != -1) L.upd(f[1], 0, g, fa);
+        if (f[2] != -1) L.upd(f[2], 0, in.op == B_ADD ? g : -g, fb);
+        break;
+      }
+      case B_NEG: {
+        const T g = L.sl(f[0], 0);
+        const bool fa = in.flags & 1;
+        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); break; }
+        if (f[1] != -1) L.upd(f[1], 0, -g, fa);
         break;
       }
       case B_MUL: {
@@ -495,28 +509,25 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         if (f[2] != -1) L.upd(f[2], 0, g * z * log(x), fb);
         break;
       }
-      case B_EXP: case B_TANH: case B_LOG: case B_ABS: case B_SQRT: case B_SIN: case B_COS: case B_POWI: {
-        T g = L.sl(f[0], 0);
-        bool fa = in.flags & 1;
-        if (f[1] == -1) break;
-        if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); break; }
-        T v;
-        switch (in.op) {
-          case B_EXP: v = g * L.ld(f[5]); break;
-          case B_TANH: { T z = L.ld(f[5]); v = g * ((T)1 - z * z); break; }
-          case B_LOG: { T x = L.ld(f[3]); v = gt_eps(x) ? g / x : (T)0; break; }
-          case B_ABS: { T x = L.ld(f[3]); v = x > (T)0 ? g : (x < (T)0 ? -g : g * (T)0); break; }
-          case B_SQRT: { T x = L.ld(f[3]); v = gt_eps(x) ? g / ((T)2 * L.ld(f[5])) : (T)0; break; }
-          case B_SIN: v = g * L.ld(f[6]); break;
-          case B_COS: v = -(g * L.ld(f[6])); break;
-          default: {  // POWI
-            int n = f[7];
-            v = n > 0 ? g * ((T)n * powi_rep(L.ld(f[3]), n - 1)) : (T)0;
-          }
-        }
-        L.upd(f[1], 0, v, fa);
-        break;
-      }
+      // unary adjoints: g times the local derivative (one case per opcode)
+#define NDVM_REV1(OPC, EXPR)                             \
+  case OPC: {                                            \
+    const T g = L.sl(f[0], 0);                           \
+    const bool fa = in.flags & 1;                        \
+    if (f[1] == -1) break;                               \
+    if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); break; } \
+    L.upd(f[1], 0, (EXPR), fa);                          \
+    break;                                               \
+  }
+      NDVM_REV1(B_EXP, g * L.ld(f[5]))
+      NDVM_REV1(B_TANH, g * ((T)1 - L.ld(f[5]) * L.ld(f[5])))
+      NDVM_REV1(B_LOG, gt_eps(L.ld(f[3])) ? g / L.ld(f[3]) : (T)0)
+      NDVM_REV1(B_ABS, L.ld(f[3]) > (T)0 ? g : (L.ld(f[3]) < (T)0 ? -g : g * (T)0))
+      NDVM_REV1(B_SQRT, gt_eps(L.ld(f[3])) ? g / ((T)2 * L.ld(f[5])) : (T)0)
+      NDVM_REV1(B_SIN, g * L.ld(f[6]))
+      NDVM_REV1(B_COS, -(g * L.ld(f[6])))
+      NDVM_REV1(B_POWI, f[7] > 0 ? g * ((T)f[7] * powi_rep(L.ld(f[3]), f[7] - 1)) : (T)0)
+#undef NDVM_REV1
       case B_SELECT: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;

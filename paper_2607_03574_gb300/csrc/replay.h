@@ -32,7 +32,7 @@ struct ReplayArgs {
 
 cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
 
-// Instructions per staged chunk (two chunk buffers of 5 KB sit after the slot file).
+// Instructions per staged chunk (two chunk buffers of 6 KB sit after the slot file).
 constexpr int kStageChunk = 128;
 
 // Size of the fixed scratch array of the no-allocation entry point (32 MiB).
