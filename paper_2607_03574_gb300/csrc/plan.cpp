@@ -15,6 +15,7 @@
 #include <climits>
 #include <cstdlib>
 #include <cstring>
+#include <map>
 #include <set>
 
 #include "cost.h"
@@ -107,6 +108,7 @@ class Planner {
   void emit_reverse(int v);
   void allocate();
   void prefetch_workspace();
+  void normalize_operands();
   int32_t encode(const PArg& a) const;
   int rev_begin_ = -1;  // first instruction of the reverse sweep
 };
@@ -530,6 +532,81 @@ void Planner::emit_region(int v) {
   emit(gr);
 }
 
+// Load-store form: every operand that slot_operand() marks is made a slot.  A
+// constant, parameter or observation is loaded once into a slot before its first
+// use -- before the enclosing data-axis loop when the use is inside one -- and the
+// slot stays live to its last use; a per-point observation is loaded inside the loop
+// body before its first use there; a workspace value not covered by the prefetch is
+// loaded right before its use.
+void Planner::normalize_operands() {
+  const int n = (int)code_.size();
+  std::vector<int> loop_of(n, -1);  // enclosing D_LOOP pc
+  for (int pc = 0, open = -1; pc < n; pc++) {
+    if (code_[pc].d.op == D_LOOP) { open = pc; continue; }
+    if (code_[pc].d.op == D_ENDLOOP) { open = -1; continue; }
+    loop_of[pc] = open;
+  }
+  std::vector<std::vector<PInst>> before(n + 1);
+  std::map<std::pair<uint32_t, int32_t>, int> uni;  // (kind, index) -> slot VR
+  std::map<int32_t, int> dob;                       // point column -> slot VR (current loop)
+  int cur_loop = -2;
+  auto load = [&](int vr, const PArg& src) {
+    PInst l;
+    l.d.op = D_LOAD;
+    l.f[0] = R(slotref(vr));
+    l.f[1] = src;
+    return l;
+  };
+  for (int pc = 0; pc < n; pc++) {
+    PInst& p = code_[pc];
+    if (loop_of[pc] != cur_loop) { dob.clear(); cur_loop = loop_of[pc]; }
+    for (int fld = 0; fld < 8; fld++) {
+      if (!slot_operand(p.d.op, fld)) continue;
+      PArg& a = p.f[fld];
+      if (!a.isref || a.r.kind == RK_SLOT) continue;
+      const uint32_t kind = a.r.kind;
+      const int32_t idx = a.r.id + a.r.off;
+      PArg src = a;
+      if (kind == RK_CONST || kind == RK_PARAM || kind == RK_OBS) {
+        auto key = std::make_pair(kind, idx);
+        auto it = uni.find(key);
+        if (it == uni.end()) {
+          int vr = new_vr(1);
+          it = uni.emplace(key, vr).first;
+          before[loop_of[pc] >= 0 ? loop_of[pc] : pc].push_back(load(vr, src));
+        }
+        a = R(slotref(it->second));
+      } else if (kind == RK_DOBS) {
+        auto it = dob.find(idx);
+        if (it == dob.end()) {
+          int vr = new_vr(1);
+          it = dob.emplace(idx, vr).first;
+          before[pc].push_back(load(vr, src));
+        }
+        a = R(slotref(it->second));
+      } else {  // workspace value outside the prefetch
+        int vr = new_vr(1);
+        before[pc].push_back(load(vr, src));
+        a = R(slotref(vr));
+      }
+    }
+  }
+  // rebuild with the loads in place and renumber the loop links
+  std::vector<PInst> out;
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < n; pc++) {
+    for (PInst& l : before[pc]) out.push_back(l);
+    newpc[pc] = (int)out.size();
+    out.push_back(code_[pc]);
+  }
+  for (PInst& p : out) {
+    if (p.d.op == D_LOOP) p.f[3] = I(newpc[p.f[3].v]);
+    if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
+  }
+  code_.swap(out);
+  if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
+}
+
 // Software pipeline for the reverse sweep of a spill tape: the scalar workspace
 // values that reverse instruction j reads are fetched (asynchronous copies into a
 // ring of slots) kFetchDepth instructions earlier, so the HBM latency overlaps the
@@ -715,6 +792,7 @@ Plan Planner::build() {
     }
   }
   if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
+  normalize_operands();
   allocate();
   pl.n_slots = n_slots_;
   pl.n_save = S_;
@@ -739,6 +817,24 @@ Plan Planner::build() {
 }
 
 }  // namespace
+
+bool slot_operand(int op, int field) {
+  switch (op) {
+    case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: case D_CMP: return field == 1 || field == 2;
+    case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: case D_SIN: case D_COS: case D_POWI:
+    case D_ACC:
+      return field == 1;
+    case D_SELECT: return field == 1 || field == 2 || field == 4;
+    case B_MUL: return field == 3 || field == 4;
+    case B_DIV: return field == 4 || field == 5;
+    case B_POW: return field == 3 || field == 4 || field == 5;
+    case B_EXP: case B_TANH: return field == 5;
+    case B_LOG: case B_ABS: case B_POWI: case B_SELECT: return field == 3;
+    case B_SQRT: return field == 3 || field == 5;
+    case B_SIN: case B_COS: return field == 6;
+    default: return false;
+  }
+}
 
 Plan make_plan(const Tape& t, bool grad, int force_mode) {
   if (force_mode == 0 || force_mode == 1) return Planner(t, grad, force_mode == 1).build();
@@ -824,6 +920,7 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
       case D_ENDLOOP: ok = f[0] == open_loop && p.code[f[0]].f[3] == (int)pc; open_loop = -1; break;
       case D_ACC: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false); break;
       case D_SEED: ok = ref_ok(f[0], 1, true); break;
+      case D_LOAD: ok = ref_ok(f[0], 1, true) && f[1] != -1 && ref_ok(f[1], 1, false); break;
       case D_LOSS: ok = ref_ok(f[0], 1, false); break;
       case B_ADD: case B_SUB: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true); break;
       case B_NEG: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true); break;
@@ -873,6 +970,8 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
         break;
       default: why = "bad opcode"; return false;
     }
+    for (int fld = 0; ok && fld < 8; fld++)
+      if (slot_operand(d.op, fld) && f[fld] != -1 && ref_kind(f[fld]) != RK_SLOT) ok = false;
     if (!ok) { why = "operand out of range at instruction " + std::to_string(pc) + " (op " + std::to_string(d.op) + ")"; return false; }
   }
   if (open_loop >= 0) { why = "unterminated loop"; return false; }

@@ -72,11 +72,17 @@ enum DOp : uint8_t {
   B_DSUM,           // f1 args offset, f2 count (args: triples target slot, first flag, partial slot)
   B_GRAD,           // grad[lane, f1] = slot f0 (or 0 if f0 < 0)
   // ---- workspace prefetch (reverse sweep of long tapes) ----
+  D_LOAD,           // slot f0 = ref f1 (a constant, parameter, observation or workspace value)
   D_FETCH,          // f1 args offset, f2 count (args: pairs workspace ref, slot ref): asynchronous
                     // copies into slots, committed as one group; flags bit0: then wait until at
                     // most kFetchDepth groups are pending
   D_NOPS
 };
+
+// Scalar instructions take slot operands only (constants, parameters, observations
+// and workspace values reach them through D_LOAD or D_FETCH); true for the operand
+// field `field` of opcode `op` whose value the kernel reads without decoding its kind.
+bool slot_operand(int op, int field);
 
 // Reverse instructions read their workspace values from slots filled this many
 // instructions ahead.

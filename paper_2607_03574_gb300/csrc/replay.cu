@@ -65,6 +65,8 @@ struct Lane {
     if (((uint32_t)ref >> 28) == RK_SLOT) return sbase[ref * ss];
     return rd(ref)[0];
   }
+  // operand of a scalar instruction: always a slot (the planner's load-store form)
+  __device__ __forceinline__ T lds(int32_t ref) const { return sbase[ref * ss]; }
   __device__ __forceinline__ bool own(int e) const { return SHARED ? ((e & emask) == eg) : true; }
   __device__ __forceinline__ int step() const { return SHARED ? emask + 1 : 1; }
   __device__ __forceinline__ int first() const { return SHARED ? eg : 0; }
@@ -290,7 +292,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
       // one case per opcode: the switch's jump is the only dispatch branch
 #define NDVM_FWD1(OPC, EXPR)                 \
   case OPC: {                                \
-    const T x = L.ld(f[1]);                  \
+    const T x = L.lds(f[1]);                 \
     const T z = (EXPR);                      \
     L.st(f[0], 0, z);                        \
     L.save_out(f[3], 0, z);                  \
@@ -298,7 +300,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
   }
 #define NDVM_FWD2(OPC, EXPR)                 \
   case OPC: {                                \
-    const T x = L.ld(f[1]), y = L.ld(f[2]);  \
+    const T x = L.lds(f[1]), y = L.lds(f[2]); \
     const T z = (EXPR);                      \
     L.st(f[0], 0, z);                        \
     L.save_out(f[3], 0, z);                  \
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
 #undef NDVM_FWD1
 #undef NDVM_FWD2
       case D_SIN: case D_COS: {
-        T x = L.ld(f[1]);
+        T x = L.lds(f[1]);
         T s = 0, c = 0;
         if (f[4] != -1 || f[5] >= 0) {
           sincos(x, &s, &c);
@@ -336,13 +338,13 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         break;
       }
       case D_POWI: {
-        T z = powi_rep(L.ld(f[1]), f[7]);
+        T z = powi_rep(L.lds(f[1]), f[7]);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
         break;
       }
       case D_CMP: {
-        T x = L.ld(f[1]), y = L.ld(f[2]);
+        T x = L.lds(f[1]), y = L.lds(f[2]);
         bool r = in.k == 0 ? x < y : in.k == 1 ? x <= y : in.k == 2 ? x > y : in.k == 3 ? x >= y : x == y;
         T z = r ? (T)1 : (T)0;
         L.st(f[0], 0, z);
@@ -350,8 +352,8 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         break;
       }
       case D_SELECT: {
-        T p = L.ld(f[1]);
-        T z = !is_zero(p) ? L.ld(f[2]) : L.ld(f[4]);
+        T p = L.lds(f[1]);
+        T z = !is_zero(p) ? L.lds(f[2]) : L.lds(f[4]);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
         break;
@@ -452,7 +454,8 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
           if (!STAGED) nxt = code[pc + 1];
         }
         break;
-      case D_ACC: L.st(f[0], 0, L.sl(f[0], 0) + L.ld(f[1])); break;
+      case D_ACC: L.st(f[0], 0, L.sl(f[0], 0) + L.lds(f[1])); break;
+      case D_LOAD: L.st(f[0], 0, L.ld(f[1])); break;
       case D_SEED: L.st(f[0], 0, (T)1); break;
       case D_GREDUCE:
         if (G > 1) {
@@ -487,24 +490,24 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
-        if (f[1] != -1) L.upd(f[1], 0, g * L.ld(f[4]), fa);
-        if (f[2] != -1) L.upd(f[2], 0, g * L.ld(f[3]), fb);
+        if (f[1] != -1) L.upd(f[1], 0, g * L.lds(f[4]), fa);
+        if (f[2] != -1) L.upd(f[2], 0, g * L.lds(f[3]), fb);
         break;
       }
       case B_DIV: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
-        T q = g / L.ld(f[4]);
+        T q = g / L.lds(f[4]);
         if (f[1] != -1) L.upd(f[1], 0, q, fa);
-        if (f[2] != -1) L.upd(f[2], 0, -(q * L.ld(f[5])), fb);
+        if (f[2] != -1) L.upd(f[2], 0, -(q * L.lds(f[5])), fb);
         break;
       }
       case B_POW: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
-        T x = L.ld(f[3]), e = L.ld(f[4]), z = L.ld(f[5]);
+        T x = L.lds(f[3]), e = L.lds(f[4]), z = L.lds(f[5]);
         if (f[1] != -1) L.upd(f[1], 0, g * e * z / x, fa);
         if (f[2] != -1) L.upd(f[2], 0, g * z * log(x), fb);
         break;
@@ -519,19 +522,19 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
     L.upd(f[1], 0, (EXPR), fa);                          \
     break;                                               \
   }
-      NDVM_REV1(B_EXP, g * L.ld(f[5]))
-      NDVM_REV1(B_TANH, g * ((T)1 - L.ld(f[5]) * L.ld(f[5])))
-      NDVM_REV1(B_LOG, gt_eps(L.ld(f[3])) ? g / L.ld(f[3]) : (T)0)
-      NDVM_REV1(B_ABS, L.ld(f[3]) > (T)0 ? g : (L.ld(f[3]) < (T)0 ? -g : g * (T)0))
-      NDVM_REV1(B_SQRT, gt_eps(L.ld(f[3])) ? g / ((T)2 * L.ld(f[5])) : (T)0)
-      NDVM_REV1(B_SIN, g * L.ld(f[6]))
-      NDVM_REV1(B_COS, -(g * L.ld(f[6])))
-      NDVM_REV1(B_POWI, f[7] > 0 ? g * ((T)f[7] * powi_rep(L.ld(f[3]), f[7] - 1)) : (T)0)
+      NDVM_REV1(B_EXP, g * L.lds(f[5]))
+      NDVM_REV1(B_TANH, g * ((T)1 - L.lds(f[5]) * L.lds(f[5])))
+      NDVM_REV1(B_LOG, gt_eps(L.lds(f[3])) ? g / L.lds(f[3]) : (T)0)
+      NDVM_REV1(B_ABS, L.lds(f[3]) > (T)0 ? g : (L.lds(f[3]) < (T)0 ? -g : g * (T)0))
+      NDVM_REV1(B_SQRT, gt_eps(L.lds(f[3])) ? g / ((T)2 * L.lds(f[5])) : (T)0)
+      NDVM_REV1(B_SIN, g * L.lds(f[6]))
+      NDVM_REV1(B_COS, -(g * L.lds(f[6])))
+      NDVM_REV1(B_POWI, f[7] > 0 ? g * ((T)f[7] * powi_rep(L.lds(f[3]), f[7] - 1)) : (T)0)
 #undef NDVM_REV1
       case B_SELECT: {
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
-        bool taken = !is_zero(L.ld(f[3]));
+        bool taken = !is_zero(L.lds(f[3]));
         if (f[1] != -1) { if (taken && !is_zero(g)) L.upd(f[1], 0, g, fa); else zero_if_first(L, f[1], 1, fa); }
         if (f[2] != -1) { if (!taken && !is_zero(g)) L.upd(f[2], 0, g, fb); else zero_if_first(L, f[2], 1, fb); }
         break;
