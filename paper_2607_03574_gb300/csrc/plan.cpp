@@ -32,6 +32,12 @@ bool prefetch_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_FMA=0 keeps the general scalar instructions instead of the fused form (a tuning knob).
+bool fma_enabled() {
+  const char* e = std::getenv("NDVM_FMA");
+  return !(e && e[0] == '0');
+}
+
 struct PRef {
   uint32_t kind = RK_SLOT;
   int32_t id = -1;  // VR id for slots; index otherwise
@@ -109,6 +115,8 @@ class Planner {
   void allocate();
   void prefetch_workspace();
   void normalize_operands();
+  void lower_fma();
+  int const_index(double v);
   int32_t encode(const PArg& a) const;
   int rev_begin_ = -1;  // first instruction of the reverse sweep
 };
@@ -532,6 +540,79 @@ void Planner::emit_region(int v) {
   emit(gr);
 }
 
+// The constant pool index holding exactly the bits of v (appended when absent).
+int Planner::const_index(double v) {
+  for (size_t k = 0; k < T.consts.size(); k++)
+    if (std::memcmp(&T.consts[k], &v, 8) == 0) return (int)k;
+  for (size_t k = 0; k < extra_consts_.size(); k++)
+    if (std::memcmp(&extra_consts_[k], &v, 8) == 0) return (int)(T.consts.size() + k);
+  extra_consts_.push_back(v);
+  return (int)(T.consts.size() + extra_consts_.size() - 1);
+}
+
+// Fused multiply-add form.  The scalar rules whose arithmetic is one product and
+// one sum become D_FMA, which the kernel executes without opcode dispatch:
+//   forward   a + b = fma(a, 1, b)      a - b = fma(-b, 1, a)
+//             a * b = fma(a, b, -0)     -a = fma(-a, 1, -0)     acc += x: fma(x, 1, acc)
+// (all exact: the product by 1 is exact, and adding -0 leaves every value,
+// including the sign of zero, unchanged), and
+//   reverse   target += g * d = fma(g, d, target) -- or fma(g, d, -0) for the first
+//             contribution -- for add, sub, neg, mul, exp, sin and cos, where the
+//             local derivative d is 1, -1, the other factor, exp(x), cos x or -sin x.
+// A reverse update is skipped when g is exactly zero (the first contribution then
+// stores -0, an exact zero), as in the general rules.  Fusing the product into the
+// accumulation rounds once where the general rules round twice.
+void Planner::lower_fma() {
+  const PArg one = R(kref(RK_CONST, one_const_));
+  const PArg mzero = R(kref(RK_CONST, const_index(-0.0)));
+  const int n = (int)code_.size();
+  std::vector<PInst> out;
+  out.reserve(n + n / 2);
+  std::vector<int> newpc(n, -1);
+  auto fma = [&](PArg dst, PArg a, bool neg, PArg b, PArg c, PArg zs, PArg save) {
+    PInst q;
+    q.d.op = D_FMA;
+    q.d.flags = neg ? 1 : 0;
+    q.f[0] = dst; q.f[1] = a; q.f[2] = b; q.f[3] = c; q.f[4] = zs; q.f[5] = save;
+    out.push_back(q);
+  };
+  for (int pc = 0; pc < n; pc++) {
+    newpc[pc] = (int)out.size();
+    const PInst& p = code_[pc];
+    const PArg* f = p.f;
+    const bool fa = p.d.flags & 1, fb = p.d.flags & 2;
+    auto upd = [&](const PArg& tgt, bool first, const PArg& g, bool neg, const PArg& d) {
+      if (tgt.isref) fma(tgt, g, neg, d, first ? mzero : tgt, g, I(-1));
+    };
+    switch (p.d.op) {
+      case D_ADD: fma(f[0], f[1], false, one, f[2], one, f[3]); break;
+      case D_SUB: fma(f[0], f[2], true, one, f[1], one, f[3]); break;
+      case D_MUL: fma(f[0], f[1], false, f[2], mzero, one, f[3]); break;
+      case D_NEG: fma(f[0], f[1], true, one, mzero, one, f[3]); break;
+      case D_ACC: fma(f[0], f[1], false, one, f[0], one, I(-1)); break;
+      case B_ADD: case B_SUB:
+        upd(f[1], fa, f[0], false, one);
+        upd(f[2], fb, f[0], p.d.op == B_SUB, one);
+        break;
+      case B_NEG: upd(f[1], fa, f[0], true, one); break;
+      case B_MUL:
+        upd(f[1], fa, f[0], false, f[4]);
+        upd(f[2], fb, f[0], false, f[3]);
+        break;
+      case B_EXP: upd(f[1], fa, f[0], false, f[5]); break;
+      case B_SIN: upd(f[1], fa, f[0], false, f[6]); break;
+      case B_COS: upd(f[1], fa, f[0], true, f[6]); break;
+      default: out.push_back(p); break;
+    }
+  }
+  for (PInst& p : out) {
+    if (p.d.op == D_LOOP) p.f[3] = I(newpc[p.f[3].v]);
+    if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
+  }
+  code_.swap(out);
+  if (rev_begin_ >= 0 && rev_begin_ < n) rev_begin_ = newpc[rev_begin_];
+}
+
 // Load-store form: every operand that slot_operand() marks is made a slot.  A
 // constant, parameter or observation is loaded once into a slot before its first
 // use -- before the enclosing data-axis loop when the use is inside one -- and the
@@ -792,6 +873,7 @@ Plan Planner::build() {
     }
   }
   if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
+  if (fma_enabled()) lower_fma();
   normalize_operands();
   allocate();
   pl.n_slots = n_slots_;
@@ -832,6 +914,7 @@ bool slot_operand(int op, int field) {
     case B_LOG: case B_ABS: case B_POWI: case B_SELECT: return field == 3;
     case B_SQRT: return field == 3 || field == 5;
     case B_SIN: case B_COS: return field == 6;
+    case D_FMA: return field >= 1 && field <= 4;
     default: return false;
   }
 }
@@ -921,6 +1004,10 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
       case D_ACC: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false); break;
       case D_SEED: ok = ref_ok(f[0], 1, true); break;
       case D_LOAD: ok = ref_ok(f[0], 1, true) && f[1] != -1 && ref_ok(f[1], 1, false); break;
+      case D_FMA:
+        ok = ref_ok(f[0], 1, true) && f[0] != -1 && save_ok(f[5], 1);
+        for (int q = 1; q <= 4; q++) ok = ok && f[q] != -1 && ref_ok(f[q], 1, true);
+        break;
       case D_LOSS: ok = ref_ok(f[0], 1, false); break;
       case B_ADD: case B_SUB: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true); break;
       case B_NEG: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true); break;

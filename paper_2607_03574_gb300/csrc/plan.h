@@ -76,6 +76,11 @@ enum DOp : uint8_t {
   D_FETCH,          // f1 args offset, f2 count (args: pairs workspace ref, slot ref): asynchronous
                     // copies into slots, committed as one group; flags bit0: then wait until at
                     // most kFetchDepth groups are pending
+  // ---- fused multiply-add form of the cheap scalar rules ----
+  D_FMA,            // slot f0 = (is_zero(slot f4) ? slot f3 : fma(+-slot f1, slot f2, slot f3)), f5 save;
+                    // flags bit0 negates the first factor.  f4 is the zero-skip test (an adjoint
+                    // whose contribution vanishes when it is exactly zero; the slot holding 1.0
+                    // when there is none)
   D_NOPS
 };
 

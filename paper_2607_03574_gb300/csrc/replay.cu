@@ -102,6 +102,14 @@ __device__ __forceinline__ bool gt_eps(float x) {
   return b > __float_as_int(1e-8f) && (b & 0x7fffffff) <= 0x7f800000;
 }
 
+// x with its sign bit flipped when neg is set (IEEE negation, exact for every value)
+__device__ __forceinline__ double flip_sign(double x, unsigned neg) {
+  return __longlong_as_double(__double_as_longlong(x) ^ ((long long)neg << 63));
+}
+__device__ __forceinline__ float flip_sign(float x, unsigned neg) {
+  return __int_as_float(__float_as_int(x) ^ (int)(neg << 31));
+}
+
 template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
   if (n == 0) return (T)1;
   T z = a;
@@ -201,7 +209,7 @@ __device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w
 // the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
 // cost while G times more warps cover the lanes.
 template <typename T, bool SHARED, bool STAGED>
-__global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
+__global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
@@ -286,6 +294,16 @@ __global__ void __launch_bounds__(256) k_replay(ReplayArgs a) {
     if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
 
     const int32_t* f = in.f;
+    if (in.op == D_FMA) {
+      // the fused form of the cheap scalar rules: no opcode dispatch
+      const T x = flip_sign(L.lds(f[1]), in.flags & 1);
+      const T c = L.lds(f[3]);
+      const T z = is_zero(L.lds(f[4])) ? c : fma(x, L.lds(f[2]), c);
+      L.st(f[0], 0, z);
+      L.save_out(f[5], 0, z);
+      if (sync_each) __syncwarp();
+      continue;
+    }
     const int w = in.r * in.c;
     switch (in.op) {
       // ------------------------------------------------------------ forward
