@@ -688,75 +688,75 @@ void Planner::normalize_operands() {
   if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
 }
 
-// Software pipeline for the reverse sweep of a spill tape: the scalar workspace
-// values that reverse instruction j reads are fetched (asynchronous copies into a
-// ring of slots) kFetchDepth instructions earlier, so the HBM latency overlaps the
-// preceding instructions instead of stalling each one.
+// Software pipeline for the reverse sweep of a spill tape.  The reverse sweep is
+// cut into windows of kFetchStride instructions; the workspace values that window k
+// reads as scalar operands are copied into a ring of slots (asynchronous copies,
+// committed as one group per window) by fetch instructions placed at the start of
+// window k - kFetchWindows, whose last one then waits until at most kFetchWindows
+// groups are pending -- so window k's values have landed when window k starts.
+// Every window commits exactly one group (possibly empty), which keeps that count
+// fixed.  The ring holds the values of any kFetchWindows + 2 consecutive windows.
 void Planner::prefetch_workspace() {
   if (rev_begin_ < 0) return;
-  auto scalar_fields = [](uint8_t op, int* fl) -> int {
-    int n = 0;
-    switch (op) {
-      case B_MUL: fl[n++] = 3; fl[n++] = 4; break;
-      case B_DIV: fl[n++] = 4; fl[n++] = 5; break;
-      case B_POW: fl[n++] = 3; fl[n++] = 4; fl[n++] = 5; break;
-      case B_EXP: case B_TANH: fl[n++] = 5; break;
-      case B_LOG: case B_ABS: case B_POWI: case B_SELECT: case B_MSCALE: fl[n++] = 3; break;
-      case B_SQRT: fl[n++] = 3; fl[n++] = 5; break;
-      case B_SIN: case B_COS: fl[n++] = 6; break;
-      case B_DET: fl[n++] = 5; break;
-      default: break;
-    }
-    return n;
-  };
-  const int nsteps = (int)code_.size() - rev_begin_;
-  std::vector<std::vector<int>> reads(nsteps);
+  const int n = (int)code_.size();
+  const int nins = n - rev_begin_;
+  const int nwin = (nins + kFetchStride - 1) / kFetchStride;
+  std::vector<std::vector<std::pair<int, int>>> uses(nwin);  // window -> (pc, field)
   size_t total = 0;
-  for (int j = 0; j < nsteps; j++) {
-    const PInst& p = code_[rev_begin_ + j];
-    int fl[4];
-    int n = scalar_fields(p.d.op, fl);
-    for (int k = 0; k < n; k++)
-      if (p.f[fl[k]].isref && p.f[fl[k]].r.kind == RK_SAVE) reads[j].push_back(fl[k]);
-    total += reads[j].size();
+  for (int pc = rev_begin_; pc < n; pc++) {
+    const PInst& p = code_[pc];
+    for (int fld = 0; fld < 8; fld++)
+      if (slot_operand(p.d.op, fld) && p.f[fld].isref && p.f[fld].r.kind == RK_SAVE) {
+        uses[(pc - rev_begin_) / kFetchStride].push_back({pc, fld});
+        total++;
+      }
   }
   if (total == 0) return;
-  // ring capacity: the most reads in flight over any kFetchDepth + 1 consecutive steps
-  int ring = 0, window = 0;
-  for (int j = 0; j < nsteps; j++) {
-    window += (int)reads[j].size();
-    if (j > kFetchDepth) window -= (int)reads[j - kFetchDepth - 1].size();
-    ring = std::max(ring, window);
+  int ring = 1;
+  for (int k = 0, run = 0; k < nwin; k++) {
+    run += (int)uses[k].size();
+    if (k >= kFetchWindows + 2) run -= (int)uses[k - kFetchWindows - 2].size();
+    ring = std::max(ring, run);
   }
-  ring += 1;
   const int ring_vr = new_vr(ring);
-  // assign ring entries in consumption order and rewrite the consumers
-  std::vector<std::vector<std::pair<PArg, PArg>>> fetch(nsteps);
+  std::vector<std::vector<std::pair<PArg, PArg>>> pairs(nwin);
   int counter = 0;
-  for (int j = 0; j < nsteps; j++) {
-    PInst& p = code_[rev_begin_ + j];
-    for (int fld : reads[j]) {
-      PArg slot = R(slotref(ring_vr, counter % ring));
-      counter++;
-      fetch[j].push_back({p.f[fld], slot});
-      p.f[fld] = slot;
+  for (int k = 0; k < nwin; k++)
+    for (auto& u : uses[k]) {
+      PArg slot = R(slotref(ring_vr, counter++ % ring));
+      PArg& fld = code_[u.first].f[u.second];
+      pairs[k].push_back({fld, slot});
+      fld = slot;
     }
-  }
-  auto fetch_inst = [&](int j, bool wait) {
-    PInst f;
-    f.d.op = D_FETCH;
-    f.d.flags = wait ? 1 : 0;
-    f.f[1] = I((int32_t)args_.size());
-    f.f[2] = I(j < nsteps ? (int32_t)fetch[j].size() : 0);
-    if (j < nsteps)
-      for (auto& pr : fetch[j]) { args_.push_back(pr.first); args_.push_back(pr.second); }
-    return f;
+  // the fetch instructions of window k: kFetchPairs copies each, the last commits
+  auto fetches = [&](int k, bool wait, std::vector<PInst>& out) {
+    const int cnt = k < nwin ? (int)pairs[k].size() : 0;
+    int e = 0;
+    do {
+      PInst f;
+      f.d.op = D_FETCH;
+      const int m = std::min(kFetchPairs, cnt - e);
+      for (int q = 0; q < m; q++) { f.f[2 * q] = pairs[k][e + q].first; f.f[2 * q + 1] = pairs[k][e + q].second; }
+      f.d.k = (uint8_t)m;
+      e += m;
+      if (e >= cnt) f.d.flags = (uint8_t)(2 | (wait ? 1 : 0));
+      out.push_back(f);
+    } while (e < cnt);
   };
   std::vector<PInst> out(code_.begin(), code_.begin() + rev_begin_);
-  for (int j = 0; j < kFetchDepth; j++) out.push_back(fetch_inst(j, false));  // prologue
-  for (int j = 0; j < nsteps; j++) {
-    out.push_back(fetch_inst(j + kFetchDepth, true));
-    out.push_back(code_[rev_begin_ + j]);
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < rev_begin_; pc++) newpc[pc] = pc;
+  for (int k = 0; k < kFetchWindows; k++) fetches(k, false, out);  // prologue
+  for (int k = 0; k < nwin; k++) {
+    fetches(k + kFetchWindows, true, out);
+    for (int pc = rev_begin_ + k * kFetchStride; pc < std::min(n, rev_begin_ + (k + 1) * kFetchStride); pc++) {
+      newpc[pc] = (int)out.size();
+      out.push_back(code_[pc]);
+    }
+  }
+  for (PInst& p : out) {
+    if (p.d.op == D_LOOP) p.f[3] = I(newpc[p.f[3].v]);
+    if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
   }
   code_.swap(out);
 }
@@ -788,7 +788,6 @@ void Planner::allocate() {
       case D_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 1; break;
       case B_GATHER: off = p.f[1].v; cnt = p.f[2].v; stride = 2; break;
       case B_DSUM: off = p.f[1].v; cnt = p.f[2].v; stride = 3; break;
-      case D_FETCH: off = p.f[1].v; cnt = p.f[2].v; stride = 2; break;
       default: break;
     }
     if (off >= 0)
@@ -872,8 +871,8 @@ Plan Planner::build() {
       emit(g);
     }
   }
-  if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
   if (fma_enabled()) lower_fma();
+  if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
   normalize_operands();
   allocate();
   pl.n_slots = n_slots_;
@@ -1049,11 +1048,10 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
         break;
       case B_GRAD: ok = ref_ok(f[0], 1, true) && f[1] >= 0 && f[1] < p.n_params; break;
       case D_FETCH:
-        ok = args_ok(f[1], f[2], 2);
-        if (ok)
-          for (int e = 0; e < f[2]; e++)
-            ok = ok && ref_kind(p.args[f[1] + 2 * e]) == RK_SAVE && ref_ok(p.args[f[1] + 2 * e], 1, false) &&
-                 ref_ok(p.args[f[1] + 2 * e + 1], 1, true);
+        ok = k <= kFetchPairs;
+        for (int e = 0; ok && e < k; e++)
+          ok = ref_kind(f[2 * e]) == RK_SAVE && ref_ok(f[2 * e], 1, false) && f[2 * e + 1] != -1 &&
+               ref_ok(f[2 * e + 1], 1, true);
         break;
       default: why = "bad opcode"; return false;
     }

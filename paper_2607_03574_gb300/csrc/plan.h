@@ -73,9 +73,10 @@ enum DOp : uint8_t {
   B_GRAD,           // grad[lane, f1] = slot f0 (or 0 if f0 < 0)
   // ---- workspace prefetch (reverse sweep of long tapes) ----
   D_LOAD,           // slot f0 = ref f1 (a constant, parameter, observation or workspace value)
-  D_FETCH,          // f1 args offset, f2 count (args: pairs workspace ref, slot ref): asynchronous
-                    // copies into slots, committed as one group; flags bit0: then wait until at
-                    // most kFetchDepth groups are pending
+  D_FETCH,          // k = count <= kFetchPairs; pairs (f0 workspace ref, f1 slot), (f2, f3), ...:
+                    // asynchronous copies into slots; flags bit1: then commit the copies issued
+                    // since the last commit as one group; bit0: then wait until at most
+                    // kFetchWindows groups are pending
   // ---- fused multiply-add form of the cheap scalar rules ----
   D_FMA,            // slot f0 = (is_zero(slot f4) ? slot f3 : fma(+-slot f1, slot f2, slot f3)), f5 save;
                     // flags bit0 negates the first factor.  f4 is the zero-skip test (an adjoint
@@ -89,9 +90,12 @@ enum DOp : uint8_t {
 // field `field` of opcode `op` whose value the kernel reads without decoding its kind.
 bool slot_operand(int op, int field);
 
-// Reverse instructions read their workspace values from slots filled this many
-// instructions ahead.
-constexpr int kFetchDepth = 8;
+// Reverse instructions read their workspace values from slots that D_FETCH fills
+// ahead of use: the reverse sweep is cut into windows of kFetchStride instructions,
+// whose values are fetched kFetchWindows windows ahead, kFetchPairs per instruction.
+constexpr int kFetchPairs = 4;
+constexpr int kFetchStride = 4;
+constexpr int kFetchWindows = 4;
 
 // 48 bytes, 16-byte aligned: the kernel fetches a record with three 128-bit loads.
 struct alignas(16) DInst {

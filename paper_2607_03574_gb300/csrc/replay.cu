@@ -65,6 +65,8 @@ struct Lane {
     if (((uint32_t)ref >> 28) == RK_SLOT) return sbase[ref * ss];
     return rd(ref)[0];
   }
+  // workspace element of this lane (a reference of kind RK_SAVE)
+  __device__ __forceinline__ const T* savep(int32_t ref) const { return save + (int64_t)(ref & kRefIndexMask) * save_ld + col; }
   // operand of a scalar instruction: always a slot (the planner's load-store form)
   __device__ __forceinline__ T lds(int32_t ref) const { return sbase[ref * ss]; }
   __device__ __forceinline__ bool own(int e) const { return SHARED ? ((e & emask) == eg) : true; }
@@ -301,6 +303,26 @@ __global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
       const T z = is_zero(L.lds(f[4])) ? c : fma(x, L.lds(f[2]), c);
       L.st(f[0], 0, z);
       L.save_out(f[5], 0, z);
+      if (sync_each) __syncwarp();
+      continue;
+    }
+    if (in.op == D_FETCH) {
+      // asynchronous copies of workspace values into slots (the owner of element 0
+      // copies; the warp barrier after the wait publishes them to the group)
+      // (unrolled: the record's fields stay in registers only when indexed by constants)
+      if (L.own(0))
+#pragma unroll
+        for (int e = 0; e < kFetchPairs; e++) {
+          if (e >= in.k) break;
+          const T* src = L.savep(f[2 * e]);
+          const unsigned dst = (unsigned)__cvta_generic_to_shared(L.wp(f[2 * e + 1]));
+          if (sizeof(T) == 8)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(src) : "memory");
+          else
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
+        }
+      if (in.flags & 2) asm volatile("cp.async.commit_group;\n" ::: "memory");
+      if (in.flags & 1) asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchWindows) : "memory");
       if (sync_each) __syncwarp();
       continue;
     }
@@ -691,23 +713,6 @@ __global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
       case B_GRAD:
         if (writer) grad[L.lane * L.P + f[1]] = f[0] == -1 ? (T)0 : L.sl(f[0], 0);
         break;
-      case D_FETCH: {
-        // asynchronous copies of workspace values into slots (the owner of element 0
-        // copies; the warp barrier after the wait publishes them to the group)
-        const int32_t* q = args + f[1];
-        if (L.own(0))
-          for (int e = 0; e < f[2]; e++) {
-            const T* src = L.rd(q[2 * e]).p;
-            const unsigned dst = (unsigned)__cvta_generic_to_shared(L.wp(q[2 * e + 1]));
-            if (sizeof(T) == 8)
-              asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(src) : "memory");
-            else
-              asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
-          }
-        asm volatile("cp.async.commit_group;\n" ::: "memory");
-        if (in.flags & 1) asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchDepth) : "memory");
-        break;
-      }
       default:
         if (a.err) atomicExch(a.err, 1);
         return;
