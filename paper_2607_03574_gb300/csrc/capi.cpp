@@ -113,6 +113,9 @@ ndvm_status device_cache(ndvm_tape* t, DevCache** out) {
 }
 
 constexpr size_t kSmemLimit = 227 * 1024;
+// lanes per launch when a workspace is used: the kernel indexes a lane's workspace
+// elements of one matrix operand with 32-bit products (element * lanes per launch)
+constexpr int64_t kMaxChunk = (int64_t)1 << 22;
 
 // Threads per lane for data-axis tapes: NDVM_THREADS_PER_LANE (1..32, a power of two)
 // overrides the default, which splits a lane's points over enough threads to give
@@ -155,13 +158,13 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     s.sstride = s.tpb;
   } else if (p.has_matrix) {
     // matrix tapes: G threads share a lane's slot column and split matrix elements;
-    // G is large enough to give every SMSP two warps and to fit two 128-thread
+    // G is large enough to give every SMSP two warps and to fit four 128-thread
     // blocks per SM in shared memory
     int g = ov > 16 ? 16 : ov;
     if (!g) {
       int gf = 1, gs = 1;
       while (gf < 16 && B * gf < 152LL * 4 * 64) gf *= 2;
-      while (gs < 16 && (size_t)p.n_slots * (128 / gs + 1) * elem > kSmemLimit / 2) gs *= 2;
+      while (gs < 16 && (size_t)p.n_slots * (128 / gs + 1) * elem > kSmemLimit / 4) gs *= 2;
       g = gf > gs ? gf : gs;
     }
     while (g < 16 && (size_t)p.n_slots * (128 / g + 1) * elem > kSmemLimit) g *= 2;
@@ -207,6 +210,7 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
     const size_t per_lane = (size_t)p.n_save * elem;
     if (!ws) return fail(NDVM_E_INVALID_ARG, "this tape needs a workspace of " + std::to_string(per_lane) + " bytes per lane");
     int64_t fit = (int64_t)(ws_bytes / per_lane);
+    if (fit > kMaxChunk) fit = kMaxChunk;
     if (fit < B) {
       fit -= fit % lanes_per_block;
       if (fit < lanes_per_block)

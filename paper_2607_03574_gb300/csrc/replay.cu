@@ -30,11 +30,55 @@
 namespace ndvm {
 namespace {
 
+// operand view: element e is p[e * s] (the host keeps e * s within 32 bits)
 template <typename T>
 struct Opnd {
   const T* p;
-  int64_t s;
-  __device__ __forceinline__ T operator[](int e) const { return p[(int64_t)e * s]; }
+  int s;
+  __device__ __forceinline__ T operator[](int e) const { return p[e * s]; }
+  __device__ __forceinline__ const T* at(int e) const { return p + e * s; }
+};
+
+// a[0] b[0] + a[sa] b[sb] + ... over n terms, accumulated left to right with fma;
+// unrolled for n <= 8 so that all operand loads issue before the chain starts
+template <typename T, int K>
+__device__ __forceinline__ T dot_fixed(const T* a, int sa, const T* b, int sb) {
+  T av[K], bv[K];
+#pragma unroll
+  for (int q = 0; q < K; q++) { av[q] = a[q * sa]; bv[q] = b[q * sb]; }
+  T s = av[0] * bv[0];
+#pragma unroll
+  for (int q = 1; q < K; q++) s = fma(av[q], bv[q], s);
+  return s;
+}
+template <typename T>
+__device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n) {
+  switch (n) {
+    case 1: return a[0] * b[0];
+    case 2: return dot_fixed<T, 2>(a, sa, b, sb);
+    case 3: return dot_fixed<T, 3>(a, sa, b, sb);
+    case 4: return dot_fixed<T, 4>(a, sa, b, sb);
+    case 5: return dot_fixed<T, 5>(a, sa, b, sb);
+    case 6: return dot_fixed<T, 6>(a, sa, b, sb);
+    case 7: return dot_fixed<T, 7>(a, sa, b, sb);
+    case 8: return dot_fixed<T, 8>(a, sa, b, sb);
+    default: {
+      T s = a[0] * b[0];
+      for (int q = 1; q < n; q++) s = fma(a[q * sa], b[q * sb], s);
+      return s;
+    }
+  }
+}
+
+// walks a thread's elements e = first, first + step, ... of a matrix with c columns
+// as (row, column) pairs without a division per element
+struct RowCol {
+  int i, j;
+  __device__ __forceinline__ RowCol(int first, int c) : i(first / c), j(first - (first / c) * c) {}
+  __device__ __forceinline__ void next(int step, int c) {
+    j += step;
+    while (j >= c) { j -= c; i++; }
+  }
 };
 
 template <typename T, bool SHARED>
@@ -57,7 +101,7 @@ struct Lane {
       case RK_CONST: return {consts + idx, 1};
       case RK_OBS: return {obs + idx, 1};
       case RK_DOBS: return {obs + dbase + idx, 1};
-      case RK_SAVE: return {save + (int64_t)idx * save_ld + col, save_ld};
+      case RK_SAVE: return {save + (int64_t)idx * save_ld + col, (int)save_ld};
       default: return {params + lane * P + idx, 1};
     }
   }
@@ -211,7 +255,7 @@ __device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w
 // the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
 // cost while G times more warps cover the lanes.
 template <typename T, bool SHARED, bool STAGED>
-__global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
+__global__ void __launch_bounds__(256, 2) k_replay(ReplayArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
@@ -429,10 +473,9 @@ __global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
       case D_MATMUL: {
         Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
         const int c = in.c, kk = in.k;
-        for (int e = L.first(); e < w; e += es) {
-          const int i = e / c, j = e - i * c;
-          T s = A[i * kk] * Bm[j];
-          for (int q = 1; q < kk; q++) s = fma(A[i * kk + q], Bm[q * c + j], s);
+        RowCol rc(L.first(), c);
+        for (int e = L.first(); e < w; e += es, rc.next(es, c)) {
+          const T s = dot(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk);
           L.st(f[0], e, s);
           L.save_out(f[3], e, s);
         }
@@ -634,21 +677,15 @@ __global__ void __launch_bounds__(256, 1) k_replay(ReplayArgs a) {
         Opnd<T> G_ = {L.wp(f[0]), L.ss};
         if (f[1] != -1) {  // gA (r x k) += gZ (r x c) * B^T (B is k x c)
           Opnd<T> Bm = L.rd(f[4]);
-          for (int e = L.first(); e < r * kk; e += es) {
-            const int i = e / kk, q = e - i * kk;
-            T s = G_[i * c] * Bm[q * c];
-            for (int j = 1; j < c; j++) s = fma(G_[i * c + j], Bm[q * c + j], s);
-            L.upd(f[1], e, s, fa);
-          }
+          RowCol rq(L.first(), kk);
+          for (int e = L.first(); e < r * kk; e += es, rq.next(es, kk))
+            L.upd(f[1], e, dot(G_.at(rq.i * c), G_.s, Bm.at(rq.j * c), Bm.s, c), fa);
         }
         if (f[2] != -1) {  // gB (k x c) += A^T (A is r x k) * gZ
           Opnd<T> A = L.rd(f[3]);
-          for (int e = L.first(); e < kk * c; e += es) {
-            const int q = e / c, j = e - q * c;
-            T s = A[q] * G_[j];
-            for (int i = 1; i < r; i++) s = fma(A[i * kk + q], G_[i * c + j], s);
-            L.upd(f[2], e, s, fb);
-          }
+          RowCol qj(L.first(), c);
+          for (int e = L.first(); e < kk * c; e += es, qj.next(es, c))
+            L.upd(f[2], e, dot(A.at(qj.i), kk * A.s, G_.at(qj.j), c * G_.s, r), fb);
         }
         break;
       }
