@@ -113,6 +113,10 @@ ndvm_status device_cache(ndvm_tape* t, DevCache** out) {
 }
 
 constexpr size_t kSmemLimit = 227 * 1024;
+// per-SM resources that bound resident blocks (sm_103a): shared memory and its
+// per-block reservation, registers, and the kernel's register cap (launch bounds)
+constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerBlockReserved = 1024;
+constexpr int kRegsPerSm = 65536, kMaxRegs = 128;
 // lanes per launch when a workspace is used: the kernel indexes a lane's workspace
 // elements of one matrix operand with 32-bit products (element * lanes per launch)
 constexpr int64_t kMaxChunk = (int64_t)1 << 22;
@@ -125,6 +129,16 @@ int threads_per_lane_override() {
     const char* e = std::getenv("NDVM_THREADS_PER_LANE");
     int g = e ? std::atoi(e) : 0;
     return (g >= 1 && g <= 32 && (g & (g - 1)) == 0) ? g : 0;
+  }();
+  return v;
+}
+
+// NDVM_STAGE=0 reads the instruction stream from global memory instead of staging
+// it through shared memory (a tuning knob).
+bool stage_enabled() {
+  static bool v = [] {
+    const char* e = std::getenv("NDVM_STAGE");
+    return !(e && e[0] == '0');
   }();
   return v;
 }
@@ -176,9 +190,17 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     s.sstride = s.tpb;
   }
   s.smem = (size_t)p.n_slots * s.sstride * elem;
-  // long loop-free streams are staged through shared memory in double-buffered chunks
+  // long loop-free streams are staged through shared memory in double-buffered chunks,
+  // unless the staging buffers would cost the launch resident blocks
   const size_t stage_bytes = 2 * kStageChunk * sizeof(DInst);
-  if (!p.has_regions && p.code.size() > 2 * (size_t)kStageChunk && s.smem + stage_bytes + 16 <= kSmemLimit) {
+  auto blocks_per_sm = [&](size_t bytes) {
+    const int by_smem = (int)(kSmemPerSm / (bytes + kSmemPerBlockReserved));
+    const int by_regs = kRegsPerSm / (kMaxRegs * s.tpb);
+    return by_smem < by_regs ? by_smem : by_regs;
+  };
+  const size_t staged_smem = (s.smem + 15) / 16 * 16 + stage_bytes;
+  if (stage_enabled() && !p.has_regions && p.code.size() > 2 * (size_t)kStageChunk && staged_smem <= kSmemLimit &&
+      blocks_per_sm(staged_smem) >= blocks_per_sm(s.smem)) {
     s.staged = 1;
     s.stage_off = (int)((s.smem + 15) / 16 * 16);
     s.smem = s.stage_off + stage_bytes;
