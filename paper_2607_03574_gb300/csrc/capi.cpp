@@ -1,6 +1,7 @@
 // C ABI implementation: tape objects, device caches, launch configuration.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -114,9 +115,11 @@ ndvm_status device_cache(ndvm_tape* t, DevCache** out) {
 
 constexpr size_t kSmemLimit = 227 * 1024;
 // per-SM resources that bound resident blocks (sm_103a): shared memory and its
-// per-block reservation, registers, and the kernel's register cap (launch bounds)
+// per-block reservation, registers, and the kernel's register caps (its launch
+// bounds: 128 per thread for the element-split and staged variants, 64 otherwise)
 constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerBlockReserved = 1024;
-constexpr int kRegsPerSm = 65536, kMaxRegs = 128;
+constexpr int kRegsPerSm = 65536, kMaxRegsStagedOrShared = 128, kMaxRegsPlain = 64;
+constexpr int64_t kNumSms = 152;
 // lanes per launch when a workspace is used: the kernel indexes a lane's workspace
 // elements of one matrix operand with 32-bit products (element * lanes per launch)
 constexpr int64_t kMaxChunk = (int64_t)1 << 22;
@@ -165,7 +168,7 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     int g = ov;
     if (!g) {
       g = 1;
-      while (g < 32 && B * g < 152LL * 512) g *= 2;
+      while (g < 32 && B * g < kNumSms * 512) g *= 2;
     }
     s.log2g = ilog2(g);
     while (s.tpb > 32 && (size_t)p.n_slots * s.tpb * elem > kSmemLimit) s.tpb /= 2;
@@ -177,7 +180,7 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     int g = ov > 16 ? 16 : ov;
     if (!g) {
       int gf = 1, gs = 1;
-      while (gf < 16 && B * gf < 152LL * 4 * 64) gf *= 2;
+      while (gf < 16 && B * gf < kNumSms * 4 * 64) gf *= 2;
       while (gs < 16 && (size_t)p.n_slots * (128 / gs + 1) * elem > kSmemLimit / 4) gs *= 2;
       g = gf > gs ? gf : gs;
     }
@@ -193,14 +196,20 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
   // long loop-free streams are staged through shared memory in double-buffered chunks,
   // unless the staging buffers would cost the launch resident blocks
   const size_t stage_bytes = 2 * kStageChunk * sizeof(DInst);
-  auto blocks_per_sm = [&](size_t bytes) {
+  auto blocks_per_sm = [&](size_t bytes, bool staged) {
     const int by_smem = (int)(kSmemPerSm / (bytes + kSmemPerBlockReserved));
-    const int by_regs = kRegsPerSm / (kMaxRegs * s.tpb);
+    const int regs = (s.shared || staged) ? kMaxRegsStagedOrShared : kMaxRegsPlain;
+    const int by_regs = kRegsPerSm / (regs * s.tpb);
     return by_smem < by_regs ? by_smem : by_regs;
   };
+  // blocks an SM would hold at most: the grid's blocks spread over the SMs
+  const int64_t lanes_per_block = s.tpb >> s.log2g;
+  const int64_t grid = (B + lanes_per_block - 1) / lanes_per_block;
+  const int want = (int)std::min<int64_t>((grid + kNumSms - 1) / kNumSms, 64);
+  auto resident = [&](size_t bytes, bool staged) { return std::min(blocks_per_sm(bytes, staged), want); };
   const size_t staged_smem = (s.smem + 15) / 16 * 16 + stage_bytes;
   if (stage_enabled() && !p.has_regions && p.code.size() > 2 * (size_t)kStageChunk && staged_smem <= kSmemLimit &&
-      blocks_per_sm(staged_smem) >= blocks_per_sm(s.smem)) {
+      resident(staged_smem, true) >= resident(s.smem, false)) {
     s.staged = 1;
     s.stage_off = (int)((s.smem + 15) / 16 * 16);
     s.smem = s.stage_off + stage_bytes;

@@ -255,7 +255,7 @@ __device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w
 // the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
 // cost while G times more warps cover the lanes.
 template <typename T, bool SHARED, bool STAGED>
-__global__ void __launch_bounds__(256, 2) k_replay(ReplayArgs a) {
+__global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(ReplayArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
