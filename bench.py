@@ -289,9 +289,15 @@ def main():
     h2d = sum(a.nbytes for a in hp) + sum(a.nbytes for a in ho)
     d2h = sum(w.B * np.dtype(npdt).itemsize * (1 + w.P) for w in progs)
 
+    hl = [torch.empty(w.B, dtype=tdt).pin_memory().numpy() for w in progs]
+    hg = [torch.empty((w.B, w.P), dtype=tdt).pin_memory().numpy() for w in progs]
+
     def e2e_step():
+        # every program's copies and replay queued on the streams, then one wait
         for k in range(len(tapes)):
-            nd.value_and_grad_host(tapes[k], hp[k], ho[k])
+            nd.value_and_grad_host_async(tapes[k], hp[k], ho[k], hl[k], hg[k], stream=side[k % len(side)])
+        for s in side:
+            s.synchronize()
 
     e2e_step()
     e2e_times = []

@@ -133,6 +133,21 @@ ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, in
                                      const void* obs, int64_t n_obs, void* loss, void* grad, void* stream);
 
 /*
+ * ndvm_value_and_grad_host_async -- ndvm_value_and_grad_host without the final
+ * synchronization: the copies and the replay are queued on `stream` and the call
+ * returns.  loss and grad hold the results once the caller has synchronized the
+ * stream; params and obs must stay unchanged until then.  Host buffers should be
+ * page-locked (cudaHostAlloc / pinned), else the copies are not asynchronous.
+ * The tape's cached device buffers are shared by its calls, so two calls on the
+ * same tape must be ordered (same stream, or a synchronization between them);
+ * calls on different tapes may overlap on different streams.  The paper has no
+ * counterpart; it lets a host-driven population of programs overlap its copies
+ * and replays.
+ */
+ndvm_status ndvm_value_and_grad_host_async(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                           const void* obs, int64_t n_obs, void* loss, void* grad, void* stream);
+
+/*
  * ndvm_value_and_grad_noalloc -- ndvm_value_and_grad for callers that may not
  * allocate device memory while they run (their device memory is planned up front
  * and must not grow).  The paper has no counterpart; this is a deployment variant.

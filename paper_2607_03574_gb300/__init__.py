@@ -63,6 +63,7 @@ def load(build_if_missing: bool = True):
             "ndvm_value_and_grad": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P, SZ, P]),
             "ndvm_value_and_grad_host": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_value_and_grad_noalloc": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
+            "ndvm_value_and_grad_host_async": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_check_device": (ctypes.c_int, [P]),
             "ndvm_launch_count": (ctypes.c_ulonglong, []),
             "ndvm_measure_fp64_peak": (ctypes.c_int, [ctypes.POINTER(ctypes.c_double), P]),
@@ -264,6 +265,25 @@ def value_and_grad_host(tape: Tape, params_np, obs_np, want_grad: bool = True, s
                                            obs_np.size, loss.ctypes.data,
                                            grad.ctypes.data if grad is not None else None, sp))
     return loss, grad
+
+
+def value_and_grad_host_async(tape: Tape, params_np, obs_np, loss_out, grad_out=None, stream=None):
+    """Queue the host-buffer computation on `stream` and return: loss_out (and grad_out)
+    hold the results after the stream is synchronized.  The arrays should be in
+    page-locked memory (e.g. views of pinned torch tensors) and must stay alive and
+    unchanged until then."""
+    import numpy as np
+    dt = F32 if params_np.dtype == np.float32 else F64
+    for a in (params_np, obs_np, loss_out) + ((grad_out,) if grad_out is not None else ()):
+        if not a.flags.c_contiguous or a.dtype != params_np.dtype:
+            raise ValueError("host buffers must be C-contiguous and of the parameters' dtype")
+    B = params_np.shape[0]
+    if loss_out.shape != (B,) or (grad_out is not None and grad_out.shape != params_np.shape):
+        raise ValueError("output shapes must be (B,) and params.shape")
+    sp = None if stream is None else ctypes.c_void_p(stream.cuda_stream)
+    _check(load().ndvm_value_and_grad_host_async(tape.handle, dt, B, params_np.ctypes.data, obs_np.ctypes.data,
+                                                 obs_np.size, loss_out.ctypes.data,
+                                                 grad_out.ctypes.data if grad_out is not None else None, sp))
 
 
 def check_device(tape: Tape):

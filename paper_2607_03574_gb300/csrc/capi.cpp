@@ -398,8 +398,13 @@ ndvm_status ndvm_value_and_grad(const ndvm_tape* tape, ndvm_dtype dtype, int64_t
   return run(const_cast<ndvm_tape*>(tape), true, dtype, B, params, obs, n_obs, loss, grad, ws, ws_bytes, stream);
 }
 
-ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
-                                     const void* obs, int64_t n_obs, void* loss, void* grad, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// host-buffer replay: copies in, replay, copies out, on one stream; `sync` waits for them
+ndvm_status host_replay(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
+                        int64_t n_obs, void* loss, void* grad, void* stream, bool sync) {
   ndvm_tape* t = const_cast<ndvm_tape*>(tape);
   if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
   if (B < 0 || n_obs < 0) return fail(NDVM_E_INVALID_ARG, "negative size");
@@ -429,8 +434,22 @@ ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, in
   if (s != NDVM_OK) return s;
   if ((e = cudaMemcpyAsync(loss, dc->h_loss, lb, cudaMemcpyDeviceToHost, st)) != cudaSuccess) return cuda_fail(e, "copy loss");
   if (want_grad && pb && (e = cudaMemcpyAsync(grad, dc->h_grad, pb, cudaMemcpyDeviceToHost, st)) != cudaSuccess) return cuda_fail(e, "copy grad");
-  if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return cuda_fail(e, "synchronize");
+  if (sync && (e = cudaStreamSynchronize(st)) != cudaSuccess) return cuda_fail(e, "synchronize");
   return NDVM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ndvm_status ndvm_value_and_grad_host(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                     const void* obs, int64_t n_obs, void* loss, void* grad, void* stream) {
+  return host_replay(tape, dtype, B, params, obs, n_obs, loss, grad, stream, true);
+}
+
+ndvm_status ndvm_value_and_grad_host_async(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params,
+                                           const void* obs, int64_t n_obs, void* loss, void* grad, void* stream) {
+  return host_replay(tape, dtype, B, params, obs, n_obs, loss, grad, stream, false);
 }
 
 ndvm_status ndvm_check_device(const ndvm_tape* tape) {

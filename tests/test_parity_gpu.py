@@ -271,3 +271,24 @@ def test_zero_adjoints_skip_infinite_factors(ndvm, oracle_mod, cuda):
     ol, og, om = oracle_run(oracle_mod, w)
     assert np.isfinite(ol).all() and np.isfinite(og).all()  # the pin: every lane stays finite
     check(gl, gg, ol, og, om)
+
+
+def test_async_host_entry_point_overlaps_tapes(ndvm, cuda):
+    """Asynchronous host-buffer calls on different tapes and streams give the
+    synchronous call's results once the streams are synchronized."""
+    import torch
+    ws = [W.logistic(B=50), W.exp_decay(B=40), W.kalman_cv4(B=30, T=12)]
+    tapes = [ndvm.trace_build(w.program, w.frontend) for w in ws]
+    streams = [torch.cuda.Stream() for _ in ws]
+    pin = lambda a: torch.tensor(a).pin_memory().numpy()
+    hp, ho = [pin(w.params) for w in ws], [pin(w.obs) for w in ws]
+    hl = [torch.empty(w.B, dtype=torch.float64).pin_memory().numpy() for w in ws]
+    hg = [torch.empty(w.params.shape, dtype=torch.float64).pin_memory().numpy() for w in ws]
+    for k in range(len(ws)):
+        ndvm.value_and_grad_host_async(tapes[k], hp[k], ho[k], hl[k], hg[k], stream=streams[k])
+    for s in streams:
+        s.synchronize()
+    for k, w in enumerate(ws):
+        sl, sg = ndvm.value_and_grad_host(tapes[k], w.params, w.obs)
+        np.testing.assert_array_equal(hl[k], sl)
+        np.testing.assert_array_equal(hg[k], sg)
