@@ -33,8 +33,45 @@ import workloads as W  # noqa: E402
 N_PROGRAMS, B_LANES, N_POINTS, SEED = 200, 4096, 256, 1234
 METRIC = "lane value+grad evals/sec (fp64, 1 GB300) and % of FP64/HBM roofline"
 UNIT = "lane-evals/s"
-WORKLOAD = (f"random-expression programs: {N_PROGRAMS} programs x {B_LANES} lanes x {N_POINTS} points, "
-            "MSE, fp64 value+grad")
+
+def measured_hbm_gbs():
+    """HBM copy bandwidth measured on the GB300s, else the recipe's fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "MEASURED_PEAKS.json hbm_gbs (measured copy)"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback 6.8 TB/s"
+
+
+def kernel_sources_digest():
+    """SHA-256 over the replay library's sources (names and bytes, sorted by name)."""
+    import hashlib
+    d = os.path.join(ROOT, "paper_2607_03574_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(d)):
+        path = os.path.join(d, name)
+        if os.path.isfile(path):
+            h.update(name.encode())
+            with open(path, "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(args, n_programs):
+    """DRAM bytes (read + write) per replay launch from the committed ncu summary of this
+    workload, if the library's sources are the ones it was taken from; else None."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if rec.get("sources_sha256") != kernel_sources_digest() or args.dtype != "f64":
+        return None
+    key = str(args.config)
+    if args.lanes or (args.config == 2 and n_programs != N_PROGRAMS):
+        return None
+    ent = rec.get("per_launch", {}).get(key)
+    return None if ent is None else float(ent["dram_bytes"])
 
 
 def dist_env():
@@ -117,25 +154,38 @@ class ClockSampler:
 def workload_for(args, seed):
     """(list of Workloads, description) of the configuration being measured."""
     if args.config == 2:
-        progs = W.random_exprs(n_programs=args.programs, B=B_LANES, n_points=N_POINTS, seed=seed)
-        return progs, WORKLOAD
-    w = W.config(args.config, seed=seed)
-    desc = {1: "exp-decay y = a exp(-b t) + c: 64 lanes x 50 points, MSE",
-            3: "logistic Euler (stack bytecode): 16384 lanes x 1000 steps, 100 obs, MSE",
-            4: "4-state constant-velocity Kalman NLL: 8192 lanes x 200 steps",
-            5: "8-state random stable Kalman NLL: 65536 lanes x 1000 steps"}[args.config]
+        B = args.lanes or B_LANES
+        progs = W.random_exprs(n_programs=args.programs, B=B, n_points=N_POINTS, seed=seed)
+        desc = (f"random-expression programs: {len(progs)} programs x {B} lanes x {N_POINTS} points, "
+                f"MSE, {args.dtype} value+grad")
+        return progs, desc
+    w = W.config(args.config, seed=seed, **({"B": args.lanes} if args.lanes else {}))
+    desc = {1: f"exp-decay y = a exp(-b t) + c: {w.B} lanes x 50 points, MSE",
+            3: f"logistic Euler (stack bytecode): {w.B} lanes x 1000 steps, 100 obs, MSE",
+            4: f"4-state constant-velocity Kalman NLL: {w.B} lanes x 200 steps",
+            5: f"8-state random stable Kalman NLL: {w.B} lanes x 1000 steps"}[args.config]
     return [w], f"{desc}, {args.dtype} value+grad"
 
 
-def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int):
+def cpu_sample_lanes(args, progs):
+    """Oracle lanes per program for a CPU sample of about 10-30 s on 16 cores."""
+    if args.cpu_lanes:
+        return min(args.cpu_lanes, progs[0].B)
+    return 2048 if args.config == 2 else progs[0].B
+
+
+def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = False):
     """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program."""
     import oracle
     oracle.build()
     t0 = time.perf_counter()
     n = 0
     for w in progs:
-        oracle.run(w.program, w.params[:lanes_per_prog], w.obs, frontend=w.frontend, nthreads=nthreads)
-        n += lanes_per_prog
+        p = w.params[:lanes_per_prog]
+        if f32:
+            p = p.astype(np.float32).astype(np.float64)
+        oracle.run(w.program, p, w.obs, frontend=w.frontend, nthreads=nthreads, f32=f32)
+        n += len(p)
     return n, time.perf_counter() - t0
 
 
@@ -144,21 +194,22 @@ def run_reference(args):
     if rank != 0:
         return 0
     cores = os.cpu_count() or 1
-    progs = W.random_exprs(n_programs=N_PROGRAMS, B=B_LANES, n_points=N_POINTS, seed=SEED)
-    lanes = args.ref_lanes
+    progs, workload = workload_for(args, SEED)
+    lanes = min(args.ref_lanes, progs[0].B)
+    f32 = args.dtype == "f32"
     for _ in range(args.warmup):
-        oracle_sample_time(progs[:4], 2, cores)
+        oracle_sample_time(progs[:4], 2, cores, f32)
     times, n = [], 0
     for _ in range(args.steps):
-        n, dt = oracle_sample_time(progs, lanes, cores)
+        n, dt = oracle_sample_time(progs, lanes, cores, f32)
         times.append(dt)
     ms = 1e3 * float(np.mean(times))
     value = n / (ms * 1e-3)
-    sample = f"{lanes} lanes of each of the {N_PROGRAMS} programs ({n} lane evals per step), all points"
+    sample = f"{lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals per step), whole data set"
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f64", "data": "synthetic", "config": {"workload": WORKLOAD, "sample": sample},
+        "dtype": args.dtype, "data": "synthetic", "config": {"workload": workload, "sample": sample},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -177,7 +228,11 @@ def main():
                     help="workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other configurations")
     ap.add_argument("--dtype", default="f64", choices=["f64", "f32"])
     ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
-    ap.add_argument("--cpu-lanes", type=int, default=1024, help="oracle lanes per program for cpu_baseline")
+    ap.add_argument("--cpu-lanes", type=int, default=0,
+                    help="oracle lanes per program for cpu_baseline (default: 2048 for the random programs, "
+                         "every lane otherwise)")
+    ap.add_argument("--lanes", type=int, default=0, help="lanes per program instead of the configuration's "
+                                                         "(smaller cases for profiling)")
     ap.add_argument("--streams", type=int, default=4, help="CUDA streams the programs are spread over")
     ap.add_argument("--no-graph", dest="graph", action="store_false",
                     help="launch every step from the host instead of replaying a captured CUDA graph")
@@ -213,9 +268,12 @@ def main():
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
     stream = torch.cuda.current_stream(dev)
     work = 0.0
+    alg_bytes = 0.0  # saved intermediates written once and read once, params, loss, grad, obs
+    esz = np.dtype(npdt).itemsize
     for tp, w in zip(tapes, progs):
         c = tp.cost()
         work += (c["work_fwd"] + c["work_rev"]) * w.B
+        alg_bytes += (2 * c["save_elems"] + 2 * w.P + 1) * esz * w.B + esz * w.obs.size
 
     # independent programs run on several streams so their kernels co-reside on the SMs
     side = [torch.cuda.Stream(dev) for _ in range(args.streams)]
@@ -307,22 +365,34 @@ def main():
         e2e_times.append(time.perf_counter() - t1)
     e2e_value = lanes_per_step / float(np.mean(e2e_times)) if world == 1 else None
 
-    # ---- roofline of the replay kernel: algorithmic FP64 work / kernel time
-    achieved = 2.0 * work / (ms * 1e-3)  # flop/s (2 per DFMA-equivalent), kernels only
+    # ---- roofline of the replay kernel: the slower of the FP64 work at the measured
+    # FP64 rate and the algorithmic bytes at the measured HBM bandwidth, against the
+    # step's kernel time (all launches of a step; they overlap on the streams)
+    achieved = 2.0 * work / (ms * 1e-3)  # flop/s (2 per DFMA-equivalent)
+    hbm_gbs, hbm_src = measured_hbm_gbs()
+    t_fp64, t_hbm = 2.0 * work / peak_flops, alg_bytes / (hbm_gbs * 1e9)
     roofline = {
         "bound": "alu", "achieved": achieved / 1e12, "peak": peak_flops / 1e12, "unit": "TFLOP/s",
-        "frac": achieved / peak_flops, "traffic": None,
+        "frac": max(t_fp64, t_hbm) / (ms * 1e-3),
+        "traffic": recorded_traffic(args, len(progs)),
         "peak_source": "FP64 FMA rate measured in this process (8 chains/thread, 4x256 threads/SM)",
         "work_dfma_per_step": work,
+        "hbm_term": {"algorithmic_bytes_per_step": alg_bytes, "peak_gbs": hbm_gbs, "peak_source": hbm_src,
+                     "ms_at_peak": 1e3 * t_hbm, "fp64_ms_at_peak": 1e3 * t_fp64,
+                     "binds": "fp64" if t_fp64 >= t_hbm else "hbm"},
     }
+    if t_hbm > t_fp64:
+        roofline.update({"bound": "hbm", "achieved": alg_bytes / (ms * 1e-3) / 1e9, "peak": hbm_gbs, "unit": "GB/s"})
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cores = os.cpu_count() or 1
-        oracle_sample_time(progs[:2], 2, cores)
-        n, dt = oracle_sample_time(progs, args.cpu_lanes, cores)
+        f32 = args.dtype == "f32"
+        lanes = cpu_sample_lanes(args, progs)
+        oracle_sample_time(progs[:2], 2, cores, f32)
+        n, dt = oracle_sample_time(progs, lanes, cores, f32)
         cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{args.cpu_lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals, {dt:.1f} s)"}
+               "sample": f"{lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals, {dt:.1f} s)"}
 
     if rank == 0:
         line = {

@@ -4,18 +4,22 @@
 //
 // Execution model.  Every lane runs the same instruction stream (the tape is
 // shared by the population), so instruction fetch and dispatch are uniform across
-// a warp; the stream is read through the read-only data path and broadcast.  A
-// group of G consecutive threads serves one lane (G = 1 except for tapes with
-// data-axis regions, where the group splits the lane's data points and reduces
-// partial sums with warp shuffles).  Each thread owns a slot file of R values in
-// shared memory, laid out [slot][thread] so a warp touches 32 consecutive
-// elements per slot.  Forward values read by the reverse sweep are either kept in
-// slots (short tapes) or stored to the workspace as [element][lane] -- each warp
-// store/load is one contiguous, coalesced run -- and read back in reverse.
+// a warp; the stream is read through L1 or, for long loop-free streams, staged in
+// shared memory in double-buffered chunks.  A group of G consecutive threads serves
+// one lane: for tapes with data-axis regions the group splits the lane's data points
+// (each thread has its own slot column; partial sums are reduced with warp
+// shuffles); for matrix tapes the group shares the lane's slot column and splits
+// each matrix instruction's elements.  Slot files live in shared memory, laid out
+// [slot][thread] (or [slot][lane]) so a warp touches consecutive elements.  Forward
+// values read by the reverse sweep are either kept in slots (short tapes) or stored
+// to the workspace as [element][lane] -- each warp store/load is one contiguous,
+// coalesced run -- and copied back into slots ahead of use in the reverse sweep.
 //
-// GB300 note: FP64 issues at about 1/73 of the FP32 rate, so the interpreter's
-// integer dispatch, shared-memory traffic and branches hide under the FP64 pipe;
-// the cost of a replay is the FP64 work it issues.
+// GB300 note: FP64 issues at about 1/73 of the FP32 rate (one warp instruction per
+// 76 cycles per scheduler), and a dependent FP64 operation waits about 64 cycles.
+// With enough warps the FP64 pipe binds; with few lanes (one warp per scheduler)
+// each lane's serial chain and the interpreter's own instructions set the time.
+// The cheap scalar rules therefore take a dispatch-free fused multiply-add path.
 #include <cuda_runtime.h>
 
 #include <cmath>
