@@ -6,6 +6,7 @@ memory and streams.  The names follow the C ABI in ``include/ndvm.h``:
 
     tape = trace_build(program_text, frontend=FE_SCHEME)
     loss, grad = value_and_grad(tape, params, obs)     # params (B, P) CUDA tensor
+    loss = loss_op(tape)(params, obs)                  # differentiable in params
 
 There is no CPU fallback: if the library is missing or the device is not a CUDA
 GPU, the calls raise.
@@ -284,6 +285,33 @@ def value_and_grad_host_async(tape: Tape, params_np, obs_np, loss_out, grad_out=
     _check(load().ndvm_value_and_grad_host_async(tape.handle, dt, B, params_np.ctypes.data, obs_np.ctypes.data,
                                                  obs_np.size, loss_out.ctypes.data,
                                                  grad_out.ctypes.data if grad_out is not None else None, sp))
+
+
+_replay_fn = None
+
+
+def loss_op(tape: Tape):
+    """The replay as a differentiable PyTorch op (the paper exposes the evaluator as one,
+    section 2): ``op(params, obs) -> loss[B]``.  Its backward returns the replay's
+    per-lane gradient scaled by the incoming per-lane cotangent (the chain rule at the
+    boundary); obs receive no gradient."""
+    global _replay_fn
+    torch = _torch()
+    if _replay_fn is None:
+        class _Replay(torch.autograd.Function):
+            @staticmethod
+            def forward(ctx, params, obs, tp):
+                loss, grad = value_and_grad(tp, params.contiguous(), obs)
+                ctx.save_for_backward(grad)
+                return loss
+
+            @staticmethod
+            def backward(ctx, gloss):
+                (grad,) = ctx.saved_tensors
+                return grad * gloss.unsqueeze(1), None, None
+
+        _replay_fn = _Replay.apply
+    return lambda params, obs: _replay_fn(params, obs, tape)
 
 
 def check_device(tape: Tape):

@@ -438,3 +438,25 @@ def test_fp32_mode_is_binary32_arithmetic(oracle_mod):
     l, g = oracle_mod.run(bc, np.array([[0.1]]), np.array([0.2]), frontend=1, f32=True)
     assert l[0] == float((f(0.1) + f(0.2)) * f(0.3))
     assert g[0, 0] == float(f(0.3))
+
+
+def test_control_fuzz_reverse_equals_dual_numbers_and_fd(oracle_mod):
+    """The oracle on the control-flow fuzz surface (let, let*, per-lane if, bounded loops,
+    data sums): its reverse mode agrees with its dual-number mode, and with central
+    differences where no lane sits near a branch switch."""
+    for w in W.control_fuzz(n_programs=12, B=4, seed=77):
+        l1, g1 = run(oracle_mod, w.program, w.params, w.obs, mode=1)
+        l2, g2 = run(oracle_mod, w.program, w.params, w.obs, mode=2)
+        np.testing.assert_array_equal(l1, l2)
+        s = np.maximum(np.max(np.abs(g1), axis=1, keepdims=True), 1e-300)
+        assert np.max(np.abs(g1 - g2) / s) < 1e-13, w.name
+    w = W.control_fuzz(n_programs=1, B=3, seed=5)[0]
+    _, g = run(oracle_mod, w.program, w.params, w.obs)
+    for k in range(w.params.shape[1]):
+        h = 1e-6
+        pp, pm = w.params.copy(), w.params.copy()
+        pp[:, k] += h
+        pm[:, k] -= h
+        lp, _ = run(oracle_mod, w.program, pp, w.obs)
+        lm, _ = run(oracle_mod, w.program, pm, w.obs)
+        np.testing.assert_allclose(g[:, k], (lp - lm) / (2 * h), rtol=1e-5, atol=1e-7)

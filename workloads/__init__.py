@@ -262,6 +262,91 @@ def random_exprs(n_programs: int = 200, B: int = 4096, n_points: int = 256, seed
 # --------------------------------------------------------------------------
 # 3. logistic growth, stack bytecode (section 7's second client)
 # --------------------------------------------------------------------------
+# ---------------------------------------------------------------- control-flow fuzz programs
+# Seeded Scheme programs over the surface a program search explores (section 6's
+# fuzzer: let, let*, per-lane if, bounded named-let loops, data sums), with the same
+# domain guards as the random expressions.  Text only: no arithmetic of the method.
+
+class _CtlGen:
+    def __init__(self, rng, n_params: int, n_points: int):
+        self.rng, self.P, self.N = rng, n_params, n_points
+        self.vars = 0
+
+    def fresh(self):
+        self.vars += 1
+        return f"v{self.vars}"
+
+    def const(self):
+        return _fmt(float(np.round(self.rng.uniform(-2, 2), 3)))
+
+    def leaf(self, env):
+        r = self.rng.random()
+        if env and r < 0.45:
+            return env[self.rng.integers(len(env))]
+        if r < 0.8:
+            return f"p{self.rng.integers(self.P)}"
+        return self.const()
+
+    def expr(self, d, env, in_sum=False):
+        if d <= 0:
+            return "(dobs 0)" if in_sum and self.rng.random() < 0.4 else self.leaf(env)
+        k = self.rng.integers(11)
+        e = lambda: self.expr(d - 1, env, in_sum)
+        if k <= 2:
+            op = ["+", "-", "*"][k]
+            return f"({op} {e()} {e()})"
+        if k == 3:
+            a = e()
+            return f"(/ {e()} (+ 1.0 (* {a} {a})))"
+        if k == 4:
+            a = e()
+            return f"(exp (/ {a} (+ 1.0 (* {a} {a}))))"
+        if k == 5:
+            a = e()
+            return f"(log (+ 1.0 (* {a} {a})))"
+        if k == 6:
+            return f"({['sin', 'cos', 'tanh'][self.rng.integers(3)]} {e()})"
+        if k == 7:
+            cmp = ["<", ">", "<=", ">="][self.rng.integers(4)]
+            return f"(if ({cmp} {e()} {e()}) {e()} {e()})"
+        if k == 8:
+            v = self.fresh()
+            return f"(let (({v} {e()})) {self.expr(d - 1, env + [v], in_sum)})"
+        if k == 9:
+            v1, v2 = self.fresh(), self.fresh()
+            b1 = e()
+            b2 = self.expr(d - 1, env + [v1], in_sum)
+            return f"(let* (({v1} {b1}) ({v2} {b2})) {self.expr(d - 1, env + [v1, v2], in_sum)})"
+        # bounded loop: a contraction keeps the accumulator in range
+        acc, i = self.fresh(), self.fresh()
+        n = int(self.rng.integers(2, 5))
+        step = self.expr(d - 1, env + [acc], in_sum)
+        return f"(let lp (({i} 0) ({acc} {e()})) (if (= {i} {n}) {acc} (lp (+ {i} 1) (* 0.5 (+ {acc} (tanh {step}))))))"
+
+
+def control_program(rng, n_params: int = 3, n_points: int = 16, depth: int = 4) -> str:
+    g = _CtlGen(rng, n_params, n_points)
+    params = " ".join(f"p{k}" for k in range(n_params))
+    lane = g.expr(depth, [])
+    body = g.expr(depth - 1, [], in_sum=True)
+    return (f"(model (params {params})\n  (+ {lane}\n     (* {_fmt(1.0 / n_points)} "
+            f"(data-sum {n_points} 1 0 (let ((r (- {body} (dobs 0)))) (* r r))))))")
+
+
+def control_fuzz(n_programs: int = 40, B: int = 96, n_params: int = 3, n_points: int = 16,
+                 seed: int = 1234) -> list:
+    """Control-flow fuzz programs: a lane-level term and a squared-residual data sum."""
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n_programs):
+        text = control_program(rng, n_params, n_points)
+        obs = rng.uniform(-2, 2, n_points)
+        params = rng.normal(0.0, 1.0, (B, n_params))
+        out.append(Workload(f"control_{i}", text, FRONTEND_SCHEME, params, obs, np.zeros(n_params),
+                            {"n_points": n_points}))
+    return out
+
+
 def logistic_bytecode(n_obs: int = 100, every: int = 10, dt: float = 0.01, x0: float = 0.1) -> str:
     lines = [
         "; logistic growth dx/dt = r x (1 - x/K), explicit Euler; MSE against observations",
