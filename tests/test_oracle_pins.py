@@ -460,3 +460,26 @@ def test_control_fuzz_reverse_equals_dual_numbers_and_fd(oracle_mod):
         lp, _ = run(oracle_mod, w.program, pp, w.obs)
         lm, _ = run(oracle_mod, w.program, pm, w.obs)
         np.testing.assert_allclose(g[:, k], (lp - lm) / (2 * h), rtol=1e-5, atol=1e-7)
+
+
+def test_second_client_workloads(oracle_mod):
+    """W1-W4 (bytecode): reverse mode equals dual numbers and central differences; W3's
+    side not taken contributes nothing (its parameter enters only through the taken side)."""
+    for w in W.second_client(B=3, seed=9):
+        l1, g1 = run(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend, mode=1)
+        l2, g2 = run(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend, mode=2)
+        np.testing.assert_array_equal(l1, l2)
+        s = np.max(np.abs(g1), axis=1, keepdims=True)
+        assert np.max(np.abs(g1 - g2) / s) < 1e-13, w.name
+        for k in range(w.P):
+            h = 1e-6 * max(1.0, float(np.abs(w.params[:, k]).max()))
+            pp, pm = w.params.copy(), w.params.copy()
+            pp[:, k] += h
+            pm[:, k] -= h
+            lp, _ = run(oracle_mod, w.program, pp, w.obs, frontend=w.frontend)
+            lm, _ = run(oracle_mod, w.program, pm, w.obs, frontend=w.frontend)
+            np.testing.assert_allclose(g1[:, k], (lp - lm) / (2 * h), rtol=1e-6, atol=1e-8, err_msg=w.name)
+    # W3 with the taken side made independent of parameter 1: its gradient is exactly zero
+    text = W.bytecode_w3(2).replace("PARAM 1\nADD\nTANH", "PUSH 0.5\nADD\nTANH")
+    _, g = run(oracle_mod, text, np.array([[0.3, 2.0], [1.0, 50.0]]), np.array([0.1, 0.2]), frontend=1)
+    np.testing.assert_array_equal(g[:, 1], 0.0)

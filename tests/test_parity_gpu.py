@@ -292,3 +292,37 @@ def test_async_host_entry_point_overlaps_tapes(ndvm, cuda):
         sl, sg = ndvm.value_and_grad_host(tapes[k], w.params, w.obs)
         np.testing.assert_array_equal(hl[k], sl)
         np.testing.assert_array_equal(hg[k], sg)
+
+
+@pytest.mark.parametrize("k", range(4), ids=["W1", "W2", "W3", "W4"])
+def test_second_client_bytecode_workloads(ndvm, oracle_mod, cuda, k):
+    """The bytecode VM's W1-W4 (scalar expression, counted loop, data-independent
+    branch, summed matrix-vector product) over 256 lanes against the oracle."""
+    w = W.second_client(B=256)[k]
+    gl, gg, fl = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(fl, gl)
+
+
+STRUCTURAL_PROGRAMS = {
+    "recursion": "(define (pw x n) (if (= n 0) 1.0 (* x (pw x (- n 1))))) (model (params a b) (+ (pw a 5) (pw b 2)))",
+    "closure": "(define (scale k) (lambda (x) (* k x))) (model (params a b) (let ((f (scale a))) (+ (f b) (f 2.0))))",
+    "lists": "(define (sum l) (if (null? l) 0.0 (+ (car l) (sum (cdr l))))) "
+             "(define (mp f l) (if (null? l) (quote ()) (cons (f (car l)) (mp f (cdr l))))) "
+             "(model (params a b) (sum (mp (lambda (x) (* x (sin x))) (list a b (* a b) 3.0))))",
+    "compose": "(define (compose f g) (lambda (x) (f (g x)))) (model (params a b) ((compose exp sin) (* a b)))",
+    "mutual": "(define (ev n x) (if (= n 0) x (od (- n 1) (* 1.5 x)))) "
+              "(define (od n x) (if (= n 0) x (ev (- n 1) (+ x (tanh x))))) (model (params a b) (ev 7 (* a b)))",
+}
+
+
+@pytest.mark.parametrize("name", sorted(STRUCTURAL_PROGRAMS))
+def test_structural_surface_programs(ndvm, oracle_mod, cuda, name):
+    """Recursion, closures, lists and higher-order functions are structural (they record
+    no tape nodes); the realized numeric trace replays to the oracle's values."""
+    rng = np.random.default_rng(3)
+    w = W.Workload(name, STRUCTURAL_PROGRAMS[name], 0, rng.uniform(-1.5, 1.5, (100, 2)), np.zeros(0), np.zeros(2))
+    gl, gg, _ = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)

@@ -195,3 +195,13 @@ def test_null_and_bad_arguments(ndvm):
     buf = ctypes.create_string_buffer(4)
     assert lib.ndvm_tape_serialize(t.handle, buf, 4, ctypes.byref(n)) == 1
     assert n.value == len(t.serialize())
+
+
+def test_structural_surface_records_only_numeric_primitives(ndvm):
+    """Recursion depth, closures and list traffic leave no trace: the tape holds the
+    leaves and one node per numeric primitive that ran."""
+    rec = "(define (pw x n) (if (= n 0) 1.0 (* x (pw x (- n 1))))) (model (params a) (pw a 5))"
+    assert ndvm.trace_build(rec).info()["n_nodes"] == 2 + 5          # 1.0, a, five products
+    lst = ("(define (sum l) (if (null? l) 0.0 (+ (car l) (sum (cdr l))))) "
+           "(model (params a b) (sum (list a b (* a b))))")
+    assert ndvm.trace_build(lst).info()["n_nodes"] == 3 + 1 + 3       # 0.0, a, b; a*b; three sums

@@ -347,6 +347,82 @@ def control_fuzz(n_programs: int = 40, B: int = 96, n_params: int = 3, n_points:
     return out
 
 
+# ---------------------------------------------------------------- second-client workloads
+# The four bytecode workloads of section 7's second client, written for this VM:
+# W1 a scalar closed-form expression, W2 a counted loop, W3 a data-independent
+# conditional (a lane mask whose predicate compares constants, so every lane takes
+# the same side), W4 a small summed matrix-vector product.  Each is fitted by
+# squared error to seeded observations.
+
+def bytecode_w1(n_obs: int = 8) -> str:
+    lines = ["; W1: y = a exp(-b t) + c sin(t), squared error at t = 0.5, 1.0, ...", "PUSH 0.0", "STORE 0"]
+    for k in range(n_obs):
+        t = _fmt(0.5 * (k + 1))
+        lines += ["PARAM 0", f"PUSH -{t}", "PARAM 1", "MUL", "EXP", "MUL", "PARAM 2", f"PUSH {t}", "SIN", "MUL",
+                  "ADD", "OBSN", "SUB", "DUP", "MUL", "LOAD 0", "ADD", "STORE 0"]
+    return "\n".join(lines + ["LOAD 0"]) + "\n"
+
+
+def bytecode_w2(steps: int = 40, every: int = 10) -> str:
+    lines = ["; W2: x' = a - b x by explicit Euler (dt 0.05), squared error every 10 steps",
+             "PUSH 0.0", "STORE 0", "PUSH 0.0", "STORE 1", f"LOOP {steps // every}", f"  LOOP {every}",
+             "    LOAD 0", "    PARAM 0", "    PARAM 1", "    LOAD 0", "    MUL", "    SUB", "    PUSH 0.05", "    MUL",
+             "    ADD", "    STORE 0", "  END", "  LOAD 0", "  OBSN", "  SUB", "  DUP", "  MUL", "  LOAD 1", "  ADD",
+             "  STORE 1", "END", "LOAD 1"]
+    return "\n".join(lines) + "\n"
+
+
+def bytecode_w3(n_obs: int = 6) -> str:
+    lines = ["; W3: a branch on a data-independent test (1 < 2): every lane takes the first side",
+             "PUSH 0.0", "STORE 0"]
+    for k in range(n_obs):
+        t = _fmt(0.25 * (k + 1))
+        lines += ["PUSH 1.0", "PUSH 2.0", "LT",
+                  "PARAM 0", f"PUSH {t}", "MUL", "PARAM 1", "ADD", "TANH",      # taken side
+                  "PARAM 1", f"PUSH {t}", "MUL", "EXP",                          # side not taken
+                  "SEL", "OBSN", "SUB", "DUP", "MUL", "LOAD 0", "ADD", "STORE 0"]
+    return "\n".join(lines + ["LOAD 0"]) + "\n"
+
+
+def bytecode_w4(n: int = 4, reps: int = 3) -> str:
+    lines = [f"; W4: sum of (A x) over {reps} observed vectors x, A = {n}x{n} parameters (row-major)",
+             "PUSH 0.0", "STORE 0"]
+    for r in range(reps):
+        lines += ["PUSH 0.0", "STORE 1"]
+        for i in range(n):
+            lines += [f"PARAM {i * n + j}" for j in range(n)]
+            lines += [f"OBS {r * (n + 1) + j}" for j in range(n)]
+            lines += [f"DOT {n}", "LOAD 1", "ADD", "STORE 1"]
+        lines += ["LOAD 1", f"OBS {r * (n + 1) + n}", "SUB", "DUP", "MUL", "LOAD 0", "ADD", "STORE 0"]
+    return "\n".join(lines + ["LOAD 0"]) + "\n"
+
+
+def second_client(B: int = 256, seed: int = 1234) -> list:
+    """W1-W4 with seeded observations and lanes around the generating parameters."""
+    rng = np.random.default_rng(seed)
+    out = []
+    t1 = 0.5 * np.arange(1, 9)
+    th1 = np.array([1.2, 0.7, 0.4])
+    obs1 = th1[0] * np.exp(-th1[1] * t1) + th1[2] * np.sin(t1) + rng.normal(0, 0.02, 8)
+    out.append(("W1", bytecode_w1(8), th1, obs1))
+    th2 = np.array([1.0, 0.8])
+    x, obs2 = 0.0, []
+    for s in range(40):
+        x = x + 0.05 * (th2[0] - th2[1] * x)
+        if (s + 1) % 10 == 0:
+            obs2.append(x + rng.normal(0, 0.01))
+    out.append(("W2", bytecode_w2(40, 10), th2, np.array(obs2)))
+    t3 = 0.25 * np.arange(1, 7)
+    th3 = np.array([0.9, -0.2])
+    out.append(("W3", bytecode_w3(6), th3, np.tanh(th3[0] * t3 + th3[1]) + rng.normal(0, 0.02, 6)))
+    th4 = rng.normal(0, 1, 16)
+    xs = rng.normal(0, 1, (3, 4))
+    obs4 = np.concatenate([np.append(x_, (th4.reshape(4, 4) @ x_).sum() + rng.normal(0, 0.05)) for x_ in xs])
+    out.append(("W4", bytecode_w4(4, 3), th4, obs4))
+    return [Workload(name, text, FRONTEND_BYTECODE, theta + rng.normal(0, 0.2, (B, theta.size)), obs, theta, {})
+            for name, text, theta, obs in out]
+
+
 def logistic_bytecode(n_obs: int = 100, every: int = 10, dt: float = 0.01, x0: float = 0.1) -> str:
     lines = [
         "; logistic growth dx/dt = r x (1 - x/K), explicit Euler; MSE against observations",
