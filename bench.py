@@ -163,7 +163,8 @@ def workload_for(args, seed):
     desc = {1: f"exp-decay y = a exp(-b t) + c: {w.B} lanes x 50 points, MSE",
             3: f"logistic Euler (stack bytecode): {w.B} lanes x 1000 steps, 100 obs, MSE",
             4: f"4-state constant-velocity Kalman NLL: {w.B} lanes x 200 steps",
-            5: f"8-state random stable Kalman NLL: {w.B} lanes x 1000 steps"}[args.config]
+            5: f"8-state random stable Kalman NLL: {w.B} lanes x 1000 steps",
+            6: f"64-state Kalman NLL population, 8-d observations: {w.B} lanes x 50 steps"}[args.config]
     return [w], f"{desc}, {args.dtype} value+grad"
 
 
@@ -224,8 +225,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
     ap.add_argument("--programs", type=int, default=N_PROGRAMS, help="programs per step (smaller for profiling)")
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5],
-                    help="workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other configurations")
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6],
+                    help="workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other configurations; "
+                         "6 a 64-state Kalman population (block-cooperative lanes)")
     ap.add_argument("--dtype", default="f64", choices=["f64", "f32"])
     ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
     ap.add_argument("--cpu-lanes", type=int, default=0,

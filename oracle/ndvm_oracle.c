@@ -1072,7 +1072,7 @@ static Val apply_prim(Ctx* cx, int p, int argc, Val* av) {
     case P_MATRIX: {
       if (argc < 2) fail(cx, "matrix needs rows and cols");
       long long r = to_int(cx, av[0], "matrix"), c = to_int(cx, av[1], "matrix");
-      if (r < 1 || c < 1 || r > 16 || c > 16) fail(cx, "matrix shape %lldx%lld outside 1..16", r, c);
+      if (r < 1 || c < 1 || r > 64 || c > 64) fail(cx, "matrix shape %lldx%lld outside 1..64", r, c);
       if (argc != 2 + r * c) fail(cx, "matrix %lldx%lld needs %lld elements, got %d", r, c, r * c, argc - 2);
       int allconst = 1;
       for (int i = 0; i < r * c; i++) {
@@ -1103,7 +1103,7 @@ static Val apply_prim(Ctx* cx, int p, int argc, Val* av) {
       long long r, c;
       if (p == P_IDENTITY) { NEED(1); r = c = to_int(cx, av[0], "identity"); }
       else { NEED(2); r = to_int(cx, av[0], "zeros"); c = to_int(cx, av[1], "zeros"); }
-      if (r < 1 || c < 1 || r > 16 || c > 16) fail(cx, "matrix shape outside 1..16");
+      if (r < 1 || c < 1 || r > 64 || c > 64) fail(cx, "matrix shape outside 1..64");
       double* v = (double*)arena_alloc(cx->ar, sizeof(double) * r * c);
       for (int i = 0; i < r; i++) for (int j = 0; j < c; j++) v[i * c + j] = (p == P_IDENTITY && i == j) ? 1.0 : 0.0;
       return mknum(const_mat(cx, (int)r, (int)c, v));

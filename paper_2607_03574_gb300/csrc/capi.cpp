@@ -120,6 +120,8 @@ constexpr size_t kSmemLimit = 227 * 1024;
 constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerBlockReserved = 1024;
 constexpr int kRegsPerSm = 65536, kMaxRegsStagedOrShared = 128, kMaxRegsPlain = 64;
 constexpr int64_t kNumSms = 152;
+// threads of a block that serves a single lane (block-cooperative matrix tapes)
+constexpr int kBlockLaneThreads = 256;
 // lanes per launch when a workspace is used: the kernel indexes a lane's workspace
 // elements of one matrix operand with 32-bit products (element * lanes per launch)
 constexpr int64_t kMaxChunk = (int64_t)1 << 22;
@@ -189,6 +191,13 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     s.log2g = ilog2(g);
     s.shared = 1;
     s.sstride = 128 / g + 1;
+    if ((size_t)p.n_slots * s.sstride * elem > kSmemLimit) {
+      // block-cooperative: one lane per block, whose threads split every matrix
+      // instruction (large state dimensions: the lane's slot file alone fills the block)
+      s.tpb = kBlockLaneThreads;
+      s.log2g = ilog2(kBlockLaneThreads);
+      s.sstride = 1;
+    }
   } else {
     while (s.tpb > 32 && (size_t)p.n_slots * s.tpb * elem > kSmemLimit) s.tpb /= 2;
     s.sstride = s.tpb;

@@ -954,7 +954,7 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
     const int32_t* f = d.f;
     const int r = d.r, c = d.c, k = d.k, w = r * c, n = d.r;
     bool ok = true;
-    if (r < 1 || c < 1 || r > 16 || c > 16 || ((d.op == D_MATMUL || d.op == B_MATMUL) && (k < 1 || k > 16)) ||
+    if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim || ((d.op == D_MATMUL || d.op == B_MATMUL) && (k < 1 || k > kMaxDim)) ||
         (d.op == D_CMP && k > 4)) {
       why = "bad shape";
       return false;
@@ -1024,7 +1024,7 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
         if (ok) for (int e = 0; e < f[2]; e++) ok = ok && ref_ok(p.args[f[1] + 2 * e], 1, true);
         break;
       case B_SCATTER:
-        ok = ref_ok(f[0], f[2], true) && ref_ok(f[1], f[4], true) && args_ok(f[3], f[2], 1) && f[4] >= 1 && f[4] <= 256;
+        ok = ref_ok(f[0], f[2], true) && ref_ok(f[1], f[4], true) && args_ok(f[3], f[2], 1) && f[4] >= 1 && f[4] <= kMaxDim * kMaxDim;
         if (ok) for (int e = 0; e < f[2]; e++) ok = ok && p.args[f[3] + e] >= 0 && p.args[f[3] + e] < f[4];
         break;
       case B_MADD: case B_MSUB: ok = ref_ok(f[0], w, true) && ref_ok(f[1], w, true) && ref_ok(f[2], w, true); break;

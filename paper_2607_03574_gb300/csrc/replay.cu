@@ -294,7 +294,14 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
   T* loss = static_cast<T*>(a.loss);
   T* grad = static_cast<T*>(a.grad);
   const bool writer = live && grank == 0;
+  // element-split groups publish each instruction's writes: a warp barrier when the
+  // group lies within a warp, a block barrier when one lane spans the whole block
   const bool sync_each = SHARED && G > 1;
+  const bool sync_block = SHARED && G > 32;
+  auto group_sync = [&]() {
+    if (sync_block) __syncthreads();
+    else __syncwarp();
+  };
   const int es = L.step();
 
   int64_t d = 0, dN = 0, dstride = 0, dbase0 = 0;
@@ -351,7 +358,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       const T z = is_zero(L.lds(f[4])) ? c : fma(x, L.lds(f[2]), c);
       L.st(f[0], 0, z);
       L.save_out(f[5], 0, z);
-      if (sync_each) __syncwarp();
+      if (sync_each) group_sync();
       continue;
     }
     if (in.op == D_FETCH) {
@@ -371,7 +378,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         }
       if (in.flags & 2) asm volatile("cp.async.commit_group;\n" ::: "memory");
       if (in.flags & 1) asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchWindows) : "memory");
-      if (sync_each) __syncwarp();
+      if (sync_each) group_sync();
       continue;
     }
     const int w = in.r * in.c;
@@ -758,7 +765,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         if (a.err) atomicExch(a.err, 1);
         return;
     }
-    if (sync_each) __syncwarp();
+    if (sync_each) group_sync();
   }
 }
 

@@ -83,7 +83,7 @@ static uint64_t const_key(int r, int c, const double* v) {
 }
 
 int Builder::konst_matrix(int r, int c, const double* v) {
-  if (r < 1 || c < 1 || r > 16 || c > 16) shape_error("constant matrix shape outside 1..16");
+  if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim) shape_error("constant matrix shape outside 1..64");
   uint64_t key = const_key(r, c, v);
   auto it = const_ids_.find(key);
   if (it != const_ids_.end()) {
@@ -112,7 +112,7 @@ int Builder::param(int k) {
 }
 
 int Builder::obs(int64_t k, int n) {
-  if (k < 0 || n < 1 || n > 16 || k > (int64_t)0x7fffffff - n) throw BuildError{NDVM_E_INVALID_ARG, "observation index out of range"};
+  if (k < 0 || n < 1 || n > kMaxDim || k > (int64_t)0x7fffffff - n) throw BuildError{NDVM_E_INVALID_ARG, "observation index out of range"};
   int64_t key = k * 32 + n;
   auto it = obs_ids_.find(key);
   if (it != obs_ids_.end()) return it->second;
@@ -168,7 +168,7 @@ int Builder::select(int p, int a, int b) {
 }
 
 int Builder::matfrom(int r, int c, const std::vector<int>& el) {
-  if (r < 1 || c < 1 || r > 16 || c > 16) shape_error("matrix shape outside 1..16");
+  if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim) shape_error("matrix shape outside 1..64");
   if ((int)el.size() != r * c) shape_error("matrix element count mismatch");
   bool allc = true;
   for (int e : el) {

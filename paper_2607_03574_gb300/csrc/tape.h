@@ -38,6 +38,10 @@ enum Op : uint16_t {
 
 const char* op_name(int op);
 
+// Largest matrix dimension (rows, columns, inner size of a product); inverse and
+// determinant take n <= 8.
+constexpr int kMaxDim = 64;
+
 // 24 bytes, serialized field by field in little-endian order.
 struct Node {
   uint16_t op = 0;

@@ -299,7 +299,7 @@ Value Tracer::apply_prim(int p, std::vector<Value>& av) {
     case PR_OBSVEC: {
       need(2);
       int64_t k = integer(av[0], "obs-vec"), n = integer(av[1], "obs-vec");
-      if (n < 1 || n > 16) unsupported("obs-vec length outside 1..16");
+      if (n < 1 || n > kMaxDim) unsupported("obs-vec length outside 1..64");
       return mknum(B.obs(k, (int)n));
     }
     case PR_CONS: need(2); return cons(av[0], av[1]);
@@ -318,7 +318,7 @@ Value Tracer::apply_prim(int p, std::vector<Value>& av) {
     case PR_MATRIX: {
       if (argc < 2) parse_error("matrix needs rows and cols");
       int64_t r = integer(av[0], "matrix"), c = integer(av[1], "matrix");
-      if (r < 1 || c < 1 || r > 16 || c > 16) throw BuildError{NDVM_E_SHAPE, "matrix shape outside 1..16"};
+      if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim) throw BuildError{NDVM_E_SHAPE, "matrix shape outside 1..64"};
       if (argc != 2 + r * c) throw BuildError{NDVM_E_SHAPE, "matrix element count mismatch"};
       std::vector<int> el(r * c);
       for (int k = 0; k < r * c; k++) el[k] = num(av[2 + k]);
@@ -338,7 +338,7 @@ Value Tracer::apply_prim(int p, std::vector<Value>& av) {
       int64_t r, c;
       if (p == PR_IDENTITY) { need(1); r = c = integer(av[0], "identity"); }
       else { need(2); r = integer(av[0], "zeros"); c = integer(av[1], "zeros"); }
-      if (r < 1 || c < 1 || r > 16 || c > 16) throw BuildError{NDVM_E_SHAPE, "matrix shape outside 1..16"};
+      if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim) throw BuildError{NDVM_E_SHAPE, "matrix shape outside 1..64"};
       std::vector<double> v(r * c, 0.0);
       if (p == PR_IDENTITY) for (int k = 0; k < r; k++) v[k * c + k] = 1.0;
       return mknum(B.konst_matrix((int)r, (int)c, v.data()));

@@ -1,0 +1,45 @@
+"""High-dimensional Kalman populations (GPU): D-state filters up to D = 64 with shared
+dynamics and observations, lanes differing in their noise parameters.  Large lanes run
+block-cooperatively (one lane per block, its threads splitting every matrix
+instruction).  Compared with the oracle at 1e-12 (conftest.rel_check)."""
+import numpy as np
+import pytest
+
+import workloads as W
+from conftest import rel_check
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu(nd, w, lanes=None):
+    import torch
+    tape = nd.trace_build(w.program, w.frontend)
+    params = w.params if lanes is None else w.params[lanes]
+    p = torch.tensor(params, device="cuda")
+    o = torch.tensor(w.obs, device="cuda")
+    loss, grad = nd.value_and_grad(tape, p, o)
+    fl = nd.forward(tape, p, o)
+    torch.cuda.synchronize()
+    nd.check_device(tape)
+    return loss.cpu().numpy(), grad.cpu().numpy(), fl.cpu().numpy()
+
+
+@pytest.mark.parametrize("D,m,T", [(12, 4, 4), (32, 8, 3), (64, 8, 2)])
+def test_highd_kalman_matches_oracle(ndvm, oracle_mod, cuda, D, m, T):
+    w = W.kalman_highd(B=20, D=D, m=m, T=T)
+    gl, gg, fl = _gpu(ndvm, w)
+    ol, og, om = oracle_mod.run(w.program, w.params, w.obs, nthreads=8, magnitudes=True)
+    ok, rep = rel_check(gl, gg, ol, og, 1e-12, om)
+    assert ok, rep
+    np.testing.assert_array_equal(fl, gl)
+
+
+def test_highd_kalman_full_size_sampled(ndvm, oracle_mod, cuda):
+    """The benchmark's configuration (D = 64, 8-d observations, T = 50, 1024 lanes),
+    four sampled lanes recomputed by the oracle."""
+    w = W.kalman_highd()
+    gl, gg, _ = _gpu(ndvm, w)
+    idx = np.array([0, 341, 682, 1023])
+    ol, og, om = oracle_mod.run(w.program, w.params[idx], w.obs, nthreads=4, magnitudes=True)
+    ok, rep = rel_check(gl[idx], gg[idx], ol, og, 1e-12, om)
+    assert ok, rep

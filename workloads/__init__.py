@@ -572,6 +572,37 @@ def kalman_rand8(B: int = 65536, T: int = 1000, seed: int = 1234, n: int = 8, m:
                     {"T": T, "n": n, "m": m, "F": F})
 
 
+def kalman_highd(B: int = 1024, D: int = 64, m: int = 8, T: int = 50, seed: int = 1234) -> Workload:
+    """A population of D-dimensional Kalman-filter likelihoods with shared dynamics,
+    observation map and observations, differing in their noise parameters (the
+    appendix's dense-numeric GPU workload, here with gradients): random transition
+    with spectral radius 0.95, H = [I_m 0], Q = exp(2 lq) I, R = exp(2 lr) I,
+    P0 = exp(2 lp0) I."""
+    rng = np.random.default_rng(seed)
+    F = random_stable_matrix(rng, D)
+    H = np.zeros((m, D))
+    H[:, :m] = np.eye(m)
+    truth = np.array([np.log(0.2), np.log(0.5), 0.0])
+    Q = np.exp(2 * truth[0]) * np.eye(D)
+    R = np.exp(2 * truth[1]) * np.eye(m)
+    P0 = np.exp(2 * truth[2]) * np.eye(D)
+    obs = _simulate_lgssm(rng, F, H, Q, R, P0, T)
+    params = truth + rng.normal(0.0, 0.3, (B, 3))
+    program = (
+        f";; {D}-state Kalman filter population, {m}-d observations, Gaussian negative log-likelihood\n"
+        f"(define F {_matrix_text(F)})\n"
+        f"(define H {_matrix_text(H)})\n"
+        + _KALMAN_LOOP.format(n=D, m=m, c=_fmt(m * math.log(2 * math.pi)))
+        + "(model (params lq lr lp0)\n"
+        f"  (kalman-nll (mscale (exp (* 2.0 lq)) (identity {D}))\n"
+        f"              (mscale (exp (* 2.0 lr)) (identity {m}))\n"
+        f"              (mscale (exp (* 2.0 lp0)) (identity {D}))\n"
+        f"              {T}))\n"
+    )
+    return Workload(f"kalman_highd{D}", program, FRONTEND_SCHEME, params, obs, truth,
+                    {"T": T, "n": D, "m": m, "F": F})
+
+
 def config(i: int, **kw):
     """Workload(s) of the five configurations at their full sizes (or overridden sizes)."""
     if i == 1:
@@ -584,4 +615,6 @@ def config(i: int, **kw):
         return kalman_cv4(**kw)
     if i == 5:
         return kalman_rand8(**kw)
+    if i == 6:
+        return kalman_highd(**kw)
     raise ValueError(i)
