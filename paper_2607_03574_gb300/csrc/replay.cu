@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
     if (sync_block) __syncthreads();
     else __syncwarp();
   };
-  const int es = L.step();
+  int es = L.step();
 
   int64_t d = 0, dN = 0, dstride = 0, dbase0 = 0;
   int loop_pc = -1;
@@ -351,6 +351,25 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
     if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
 
     const int32_t* f = in.f;
+    if (in.op == 0 || in.op >= D_NOPS) {  // not an opcode: every thread stops together
+      if (a.err && tid == 0) atomicExch(a.err, 1);
+      return;
+    }
+    if (sync_block) {
+      // a lane spread over the whole block: instructions over many elements use every
+      // thread; the rest (scalars, small inverses and determinants, fetches) run in
+      // warp 0 alone, with ownership narrowed to its 32 threads, while the other warps
+      // wait at the barrier that ends the instruction
+      const bool wide = in.op == D_GATHER || in.op == D_MADD || in.op == D_MSUB || in.op == D_MSCALE ||
+                        in.op == D_MATMUL || in.op == D_ZERO || in.op == B_MADD || in.op == B_MSUB ||
+                        in.op == B_MSCALE || in.op == B_MATMUL || in.op == B_SCATTER;
+      if (!wide && (tid >> 5) != 0) {
+        group_sync();
+        continue;
+      }
+      L.emask = wide ? G - 1 : 31;
+      es = L.step();
+    }
     if (in.op == D_FMA) {
       // the fused form of the cheap scalar rules: no opcode dispatch
       const T x = flip_sign(L.lds(f[1]), in.flags & 1);
@@ -763,6 +782,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         break;
       default:
         if (a.err) atomicExch(a.err, 1);
+        if (sync_block) break;  // warp 0 alone may be here: keep the barrier count, stop nothing
         return;
     }
     if (sync_each) group_sync();
