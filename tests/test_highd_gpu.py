@@ -43,3 +43,37 @@ def test_highd_kalman_full_size_sampled(ndvm, oracle_mod, cuda):
     ol, og, om = oracle_mod.run(w.program, w.params[idx], w.obs, nthreads=4, magnitudes=True)
     ok, rep = rel_check(gl[idx], gg[idx], ol, og, 1e-12, om)
     assert ok, rep
+
+
+def test_highd_block_lanes_decompose_and_chunk(ndvm, cuda):
+    """Block-cooperative lanes: a lane replayed alone, or in workspace chunks of a few
+    lanes, gives the batched result bit for bit."""
+    import torch
+    w = W.kalman_highd(B=9, D=32, m=8, T=3)
+    tape = ndvm.trace_build(w.program, w.frontend)
+    p = torch.tensor(w.params, device="cuda")
+    o = torch.tensor(w.obs, device="cuda")
+    bl, bg = ndvm.value_and_grad(tape, p, o)
+    per_lane = tape.workspace_bytes(1, 0)
+    cl, cg = ndvm.value_and_grad(tape, p, o, ws_bytes=2 * per_lane + 8)  # chunks of two lanes
+    sl, sg = ndvm.value_and_grad(tape, p[4:5].contiguous(), o)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(cl.cpu().numpy(), bl.cpu().numpy())
+    np.testing.assert_array_equal(cg.cpu().numpy(), bg.cpu().numpy())
+    np.testing.assert_array_equal(sl.cpu().numpy()[0], bl.cpu().numpy()[4])
+    np.testing.assert_array_equal(sg.cpu().numpy()[0], bg.cpu().numpy()[4])
+
+
+def test_highd_fp32_variant(ndvm, oracle_mod, cuda):
+    """fp32 replay of a 32-state population against the oracle in binary32, 1e-5."""
+    import torch
+    w = W.kalman_highd(B=12, D=32, m=8, T=3)
+    w.params = w.params.astype(np.float32).astype(np.float64)
+    tape = ndvm.trace_build(w.program, w.frontend)
+    p = torch.tensor(w.params, dtype=torch.float32, device="cuda")
+    o = torch.tensor(w.obs, dtype=torch.float32, device="cuda")
+    gl, gg = ndvm.value_and_grad(tape, p, o)
+    torch.cuda.synchronize()
+    ol, og, om = oracle_mod.run(w.program, w.params, w.obs, nthreads=8, magnitudes=True, f32=True)
+    ok, rep = rel_check(gl.double().cpu().numpy(), gg.double().cpu().numpy(), ol, og, 1e-5, om)
+    assert ok, rep
