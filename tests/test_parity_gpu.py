@@ -326,3 +326,39 @@ def test_structural_surface_programs(ndvm, oracle_mod, cuda, name):
     gl, gg, _ = gpu_run(ndvm, w)
     ol, og, om = oracle_run(oracle_mod, w)
     check(gl, gg, ol, og, om)
+
+
+def test_degenerate_programs(ndvm, oracle_mod, cuda):
+    """A parameter that the trace never reaches has an exactly zero gradient; a program
+    without parameters has a loss and no gradient columns; a constant program gives the
+    constant on every lane."""
+    import torch
+    w = W.Workload("unused", "(model (params a b c) (* (sin a) (exp c)))", 0,
+                   np.random.default_rng(1).normal(size=(37, 3)), np.zeros(0), np.zeros(3))
+    gl, gg, _ = gpu_run(ndvm, w)
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, om)
+    np.testing.assert_array_equal(gg[:, 1], 0.0)
+    t0 = ndvm.trace_build("(model (params) (* 2.0 (+ 1.5 (obs 0))))")
+    p0 = torch.zeros((5, 0), dtype=torch.float64, device="cuda")
+    o0 = torch.tensor([0.25], dtype=torch.float64, device="cuda")
+    l0, g0 = ndvm.value_and_grad(t0, p0, o0)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(l0.cpu().numpy(), np.full(5, 3.5))
+    assert g0.shape == (5, 0)
+    tc = ndvm.trace_build("(model (params a) 4.25)")
+    lc, gc = ndvm.value_and_grad(tc, torch.ones((3, 1), dtype=torch.float64, device="cuda"), None)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(lc.cpu().numpy(), np.full(3, 4.25))
+    np.testing.assert_array_equal(gc.cpu().numpy(), 0.0)
+
+
+def test_million_lanes_sampled(ndvm, oracle_mod, cuda):
+    """2^20 lanes in one call (8192 blocks): sampled lanes against the oracle."""
+    rng = np.random.default_rng(8)
+    base = W.exp_decay(B=1)
+    w = W.Workload("big", base.program, 0, 1.0 + 0.3 * rng.standard_normal((1 << 20, 3)), base.obs, base.truth)
+    gl, gg, _ = gpu_run(ndvm, w)
+    idx = np.array([0, 1, 12345, 524287, 524288, (1 << 20) - 1])
+    ol, og, om = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, om)
