@@ -97,7 +97,7 @@ constexpr int kFetchPairs = 4;
 constexpr int kFetchStride = 4;
 constexpr int kFetchWindows = 4;
 
-// 48 bytes, 16-byte aligned: the kernel fetches a record with three 128-bit loads.
+// 48 bytes, 16-byte aligned (three 128-bit words; staged copies move 16-byte pieces).
 struct alignas(16) DInst {
   uint8_t op = 0, r = 1, c = 1, k = 1;
   uint8_t flags = 0, pad0 = 0, pad1 = 0, pad2 = 0;
