@@ -32,6 +32,49 @@ bool prefetch_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_PAIR=0 keeps adjacent independent fused instructions in separate records.
+bool pair_enabled() {
+  const char* e = std::getenv("NDVM_PAIR");
+  return !(e && e[0] == '0');
+}
+
+// Two adjacent D_FMA records without saves, where the second neither reads the first's
+// result nor shares its destination, become one D_FMA2: one dispatch, both products in
+// flight together.  Runs on the encoded stream (physical slots): the kernel loads every
+// operand of the pair before it stores either result, so a second destination that
+// the first instruction reads is also safe.
+void pair_fma(Plan& pl) {
+  const int n = (int)pl.code.size();
+  std::vector<DInst> out;
+  out.reserve(n);
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < n; pc++) {
+    const DInst& a = pl.code[pc];
+    newpc[pc] = (int)out.size();
+    if (pc + 1 < n && a.op == D_FMA && pl.code[pc + 1].op == D_FMA && a.f[5] == -1 && pl.code[pc + 1].f[5] == -1) {
+      const DInst& b = pl.code[pc + 1];
+      const bool raw = b.f[1] == a.f[0] || b.f[2] == a.f[0] || b.f[3] == a.f[0] || b.f[4] == a.f[0];
+      if (!raw && b.f[0] != a.f[0]) {
+        DInst q;
+        q.op = D_FMA2;
+        q.flags = (uint8_t)((a.flags & 1) | ((b.flags & 1) << 1));
+        for (int k = 0; k < 5; k++) q.f[k] = a.f[k];
+        q.f[5] = b.f[0]; q.f[6] = b.f[1]; q.f[7] = b.f[2]; q.pad3 = b.f[3]; q.pad4 = b.f[4];
+        out.push_back(q);
+        newpc[pc + 1] = newpc[pc];
+        pc++;
+        continue;
+      }
+    }
+    out.push_back(a);
+  }
+  for (DInst& d : out) {
+    if (d.op == D_LOOP) d.f[3] = newpc[d.f[3]];
+    if (d.op == D_ENDLOOP) d.f[0] = newpc[d.f[0]];
+  }
+  pl.code.swap(out);
+}
+
 // NDVM_FMA=0 keeps the general scalar instructions instead of the fused form (a tuning knob).
 bool fma_enabled() {
   const char* e = std::getenv("NDVM_FMA");
@@ -886,6 +929,7 @@ Plan Planner::build() {
     pl.code.push_back(d);
   }
   for (const PArg& a : args_) pl.args.push_back(encode(a));
+  if (fma_enabled() && pair_enabled()) pair_fma(pl);
   for (const DInst& d : pl.code)
     if (d.op == D_MATMUL || d.op == D_MADD || d.op == D_MSUB || d.op == D_MSCALE || d.op == D_INV ||
         ((d.op == D_DET || d.op == D_LOGDET) && d.r > 1) || (d.op == D_GATHER && d.f[2] > 1))
@@ -1003,6 +1047,12 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
       case D_ACC: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false); break;
       case D_SEED: ok = ref_ok(f[0], 1, true); break;
       case D_LOAD: ok = ref_ok(f[0], 1, true) && f[1] != -1 && ref_ok(f[1], 1, false); break;
+      case D_FMA2:
+        ok = f[0] != -1 && f[5] != -1 && ref_ok(f[0], 1, true) && ref_ok(f[5], 1, true);
+        for (int q = 1; q <= 4; q++) ok = ok && f[q] != -1 && ref_ok(f[q], 1, true);
+        ok = ok && f[6] != -1 && f[7] != -1 && d.pad3 != -1 && d.pad4 != -1 && ref_ok(f[6], 1, true) &&
+             ref_ok(f[7], 1, true) && ref_ok(d.pad3, 1, true) && ref_ok(d.pad4, 1, true);
+        break;
       case D_FMA:
         ok = ref_ok(f[0], 1, true) && f[0] != -1 && save_ok(f[5], 1);
         for (int q = 1; q <= 4; q++) ok = ok && f[q] != -1 && ref_ok(f[q], 1, true);

@@ -82,6 +82,9 @@ enum DOp : uint8_t {
                     // flags bit0 negates the first factor.  f4 is the zero-skip test (an adjoint
                     // whose contribution vanishes when it is exactly zero; the slot holding 1.0
                     // when there is none)
+  D_FMA2,           // two independent D_FMA without saves in one record: (f0 dst, f1, f2, f3, f4 zero-skip)
+                    // and (f5 dst, f6, f7, pad3, pad4 zero-skip); flags bit0 / bit1 negate the first
+                    // factor of the first / second
   D_NOPS
 };
 

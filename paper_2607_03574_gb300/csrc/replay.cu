@@ -380,6 +380,18 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       if (sync_each) group_sync();
       continue;
     }
+    if (in.op == D_FMA2) {
+      // two independent fused updates: every operand is loaded before either store
+      const T x1 = flip_sign(L.lds(f[1]), in.flags & 1), y1 = L.lds(f[2]), c1 = L.lds(f[3]), g1 = L.lds(f[4]);
+      const T x2 = flip_sign(L.lds(f[6]), (in.flags >> 1) & 1), y2 = L.lds(f[7]), c2 = L.lds(in.pad3),
+              g2 = L.lds(in.pad4);
+      const T z1 = is_zero(g1) ? c1 : fma(x1, y1, c1);
+      const T z2 = is_zero(g2) ? c2 : fma(x2, y2, c2);
+      L.st(f[0], 0, z1);
+      L.st(f[5], 0, z2);
+      if (sync_each) group_sync();
+      continue;
+    }
     if (in.op == D_FETCH) {
       // asynchronous copies of workspace values into slots (the owner of element 0
       // copies; the warp barrier after the wait publishes them to the group)
