@@ -117,6 +117,7 @@ class Planner {
   int N = 0;
   std::vector<uint8_t> active_, region_body_;
   std::vector<char> need_val_, need_aux_;
+  std::vector<int> twin_inv_;  // DET/LOGDET node -> an INV node of the same matrix (or -1)
   std::vector<int> val_vr_, aux_vr_, adj_vr_;
   std::vector<int64_t> save_, aux_save_;
   std::vector<VR> vrs_;
@@ -222,6 +223,7 @@ void Planner::analyze() {
   }
   need_val_.assign(N, 0);
   need_aux_.assign(N, 0);
+  twin_inv_.assign(N, -1);
   if (grad_) {
     for (int v = 0; v < N; v++) {
       if (!active_[v]) continue;
@@ -242,6 +244,21 @@ void Planner::analyze() {
         case OP_LOGDET: need_aux_[v] = 1; break;
         default: break;
       }
+    }
+    // a determinant whose matrix is also inverted by the program (a Kalman filter
+    // takes both of its innovation covariance) reads that inverse in the reverse sweep
+    // instead of computing its own: the forward sweep then finds the determinant only
+    std::map<int, int> inv_of;
+    for (int v = 0; v < N; v++)
+      if (T.nodes[v].op == OP_INV && active_[v] && !region_body_[v]) inv_of.emplace(T.nodes[v].a, v);
+    for (int v = 0; v < N; v++) {
+      const Node& n = T.nodes[v];
+      if ((n.op != OP_DET && n.op != OP_LOGDET) || !need_aux_[v] || region_body_[v]) continue;
+      auto it = inv_of.find(n.a);
+      if (it == inv_of.end()) continue;
+      twin_inv_[v] = it->second;
+      need_aux_[v] = 0;
+      need_val_[it->second] = 1;
     }
   }
   val_vr_.assign(N, -1);
@@ -479,9 +496,12 @@ void Planner::emit_reverse(int v) {
     case OP_INV: p.d.op = B_INV; p.d.r = T.nodes[n.a].rows; tgt(n.a, 1, 0); p.f[5] = R(rref(v)); break;
     case OP_DET:
       p.d.op = B_DET; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0);
-      p.f[5] = R(rref(v)); p.f[6] = R(rauxref(v));
+      p.f[5] = R(rref(v)); p.f[6] = R(twin_inv_[v] >= 0 ? rref(twin_inv_[v]) : rauxref(v));
       break;
-    case OP_LOGDET: p.d.op = B_LOGDET; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0); p.f[6] = R(rauxref(v)); break;
+    case OP_LOGDET:
+      p.d.op = B_LOGDET; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0);
+      p.f[6] = R(twin_inv_[v] >= 0 ? rref(twin_inv_[v]) : rauxref(v));
+      break;
     case OP_TRACE: p.d.op = B_TRACE; p.d.r = T.nodes[n.a].rows; p.d.c = 1; tgt(n.a, 1, 0); break;
     case OP_DSUM: {
       p.d.op = B_DSUM;
