@@ -34,6 +34,7 @@ ndvm_status cuda_fail(cudaError_t e, const char* where) {
 
 struct DevPlan {
   DInst* code = nullptr;
+  DInst* code_paired = nullptr;  // the paired stream (staged and element-split variants), or null
   int32_t* args = nullptr;
   double* consts_d = nullptr;
   float* consts_f = nullptr;
@@ -63,7 +64,7 @@ struct ndvm_tape {
 namespace {
 
 void free_plan(DevPlan& p) {
-  cudaFree(p.code); cudaFree(p.args); cudaFree(p.consts_d); cudaFree(p.consts_f);
+  cudaFree(p.code); cudaFree(p.code_paired); cudaFree(p.args); cudaFree(p.consts_d); cudaFree(p.consts_f);
   p = DevPlan{};
 }
 
@@ -82,6 +83,11 @@ ndvm_status upload_plan(const Tape& t, const Plan& p, DevPlan& d) {
   if ((e = cudaMalloc(&d.consts_f, sizeof(float) * cf.size())) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
   if (!p.code.empty() && (e = cudaMemcpy(d.code, p.code.data(), sizeof(DInst) * p.code.size(), cudaMemcpyHostToDevice)) != cudaSuccess)
     return cuda_fail(e, "cudaMemcpy");
+  if (!p.code_paired.empty()) {
+    if ((e = cudaMalloc(&d.code_paired, sizeof(DInst) * (p.code_paired.size() + 1))) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
+    if ((e = cudaMemcpy(d.code_paired, p.code_paired.data(), sizeof(DInst) * p.code_paired.size(), cudaMemcpyHostToDevice)) != cudaSuccess)
+      return cuda_fail(e, "cudaMemcpy");
+  }
   if ((e = cudaMemcpy(d.args, args.data(), sizeof(int32_t) * args.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
   if ((e = cudaMemcpy(d.consts_d, c.data(), sizeof(double) * c.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
   if ((e = cudaMemcpy(d.consts_f, cf.data(), sizeof(float) * cf.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
@@ -264,8 +270,11 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   if (s != NDVM_OK) return s;
   const DevPlan& dp = grad ? dc->grad : dc->value;
   ReplayArgs a;
-  a.code = dp.code;
-  a.n_code = (int)p.code.size();
+  // the staged and element-split variants run the paired stream; the plain one does not
+  // carry the paired instruction (it would cost its register budget)
+  const bool paired = (sh.staged || sh.shared) && dp.code_paired != nullptr;
+  a.code = paired ? dp.code_paired : dp.code;
+  a.n_code = (int)(paired ? p.code_paired.size() : p.code.size());
   a.args = dp.args;
   a.consts = dtype == NDVM_F32 ? (const void*)dp.consts_f : (const void*)dp.consts_d;
   a.obs = obs;
@@ -543,8 +552,9 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   cudaError_t e = noalloc_scratch(&scratch);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
   ReplayArgs a;
-  a.code = dc->grad.code;
-  a.n_code = (int)p.code.size();
+  const bool paired = (sh.staged || sh.shared) && dc->grad.code_paired != nullptr;
+  a.code = paired ? dc->grad.code_paired : dc->grad.code;
+  a.n_code = (int)(paired ? p.code_paired.size() : p.code.size());
   a.args = dc->grad.args;
   a.consts = dtype == NDVM_F32 ? (const void*)dc->grad.consts_f : (const void*)dc->grad.consts_d;
   a.obs = obs;

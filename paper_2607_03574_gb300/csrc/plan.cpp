@@ -43,16 +43,16 @@ bool pair_enabled() {
 // flight together.  Runs on the encoded stream (physical slots): the kernel loads every
 // operand of the pair before it stores either result, so a second destination that
 // the first instruction reads is also safe.
-void pair_fma(Plan& pl) {
-  const int n = (int)pl.code.size();
+std::vector<DInst> pair_fma(const std::vector<DInst>& code) {
+  const int n = (int)code.size();
   std::vector<DInst> out;
   out.reserve(n);
   std::vector<int> newpc(n, -1);
   for (int pc = 0; pc < n; pc++) {
-    const DInst& a = pl.code[pc];
+    const DInst& a = code[pc];
     newpc[pc] = (int)out.size();
-    if (pc + 1 < n && a.op == D_FMA && pl.code[pc + 1].op == D_FMA && a.f[5] == -1 && pl.code[pc + 1].f[5] == -1) {
-      const DInst& b = pl.code[pc + 1];
+    if (pc + 1 < n && a.op == D_FMA && code[pc + 1].op == D_FMA && a.f[5] == -1 && code[pc + 1].f[5] == -1) {
+      const DInst& b = code[pc + 1];
       const bool raw = b.f[1] == a.f[0] || b.f[2] == a.f[0] || b.f[3] == a.f[0] || b.f[4] == a.f[0];
       if (!raw && b.f[0] != a.f[0]) {
         DInst q;
@@ -72,7 +72,7 @@ void pair_fma(Plan& pl) {
     if (d.op == D_LOOP) d.f[3] = newpc[d.f[3]];
     if (d.op == D_ENDLOOP) d.f[0] = newpc[d.f[0]];
   }
-  pl.code.swap(out);
+  return out;
 }
 
 // NDVM_FMA=0 keeps the general scalar instructions instead of the fused form (a tuning knob).
@@ -949,7 +949,7 @@ Plan Planner::build() {
     pl.code.push_back(d);
   }
   for (const PArg& a : args_) pl.args.push_back(encode(a));
-  if (fma_enabled() && pair_enabled()) pair_fma(pl);
+  if (fma_enabled() && pair_enabled()) pl.code_paired = pair_fma(pl.code);
   for (const DInst& d : pl.code)
     if (d.op == D_MATMUL || d.op == D_MADD || d.op == D_MSUB || d.op == D_MSCALE || d.op == D_INV ||
         ((d.op == D_DET || d.op == D_LOGDET) && d.r > 1) || (d.op == D_GATHER && d.f[2] > 1))
@@ -989,7 +989,14 @@ Plan make_plan(const Tape& t, bool grad, int force_mode) {
   return Planner(t, grad, true).build();
 }
 
+bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_consts, std::string& why);
+
 bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
+  return validate_code(p, p.code, n_consts, why) &&
+         (p.code_paired.empty() || validate_code(p, p.code_paired, n_consts, why));
+}
+
+bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_consts, std::string& why) {
   const size_t nconst = n_consts + p.extra_consts.size();
   // ref: any readable operand; slot: a writable slot reference
   auto ref_ok = [&](int32_t r, int64_t width, bool must_slot) -> bool {
@@ -1013,8 +1020,8 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
     return off >= 0 && cnt >= 0 && (size_t)off + (size_t)cnt * stride <= p.args.size();
   };
   int open_loop = -1;
-  for (size_t pc = 0; pc < p.code.size(); pc++) {
-    const DInst& d = p.code[pc];
+  for (size_t pc = 0; pc < code.size(); pc++) {
+    const DInst& d = code[pc];
     const int32_t* f = d.f;
     const int r = d.r, c = d.c, k = d.k, w = r * c, n = d.r;
     bool ok = true;
@@ -1059,11 +1066,11 @@ bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
       case D_TRACE: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, false); break;
       case D_ZERO: case D_GREDUCE: ok = f[1] >= 0 && ref_ok(f[0], f[1], true); break;
       case D_LOOP:
-        ok = open_loop < 0 && f[3] > (int)pc && f[3] < (int)p.code.size() && p.code[f[3]].op == D_ENDLOOP &&
+        ok = open_loop < 0 && f[3] > (int)pc && f[3] < (int)code.size() && code[f[3]].op == D_ENDLOOP &&
              f[0] >= 0 && f[1] >= 0 && f[2] >= 0;
         open_loop = (int)pc;
         break;
-      case D_ENDLOOP: ok = f[0] == open_loop && p.code[f[0]].f[3] == (int)pc; open_loop = -1; break;
+      case D_ENDLOOP: ok = f[0] == open_loop && code[f[0]].f[3] == (int)pc; open_loop = -1; break;
       case D_ACC: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false); break;
       case D_SEED: ok = ref_ok(f[0], 1, true); break;
       case D_LOAD: ok = ref_ok(f[0], 1, true) && f[1] != -1 && ref_ok(f[1], 1, false); break;

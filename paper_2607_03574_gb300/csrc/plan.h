@@ -120,6 +120,9 @@ struct Plan {
   int64_t n_obs_min = 0;
   int32_t max_dobs = -1;      // largest DOBS column read (for validation)
   std::vector<DInst> code;
+  // the same stream with adjacent independent D_FMA paired into D_FMA2 (for the staged
+  // and element-split kernel variants; the plain variant runs `code`)
+  std::vector<DInst> code_paired;
   std::vector<int32_t> args;
   std::vector<double> extra_consts;  // appended after the tape's constant pool
   // algorithmic cost per lane (for the roofline): DFMA-equivalents and saved bytes

@@ -380,8 +380,9 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       if (sync_each) group_sync();
       continue;
     }
-    if (in.op == D_FMA2) {
+    if ((SHARED || STAGED) && in.op == D_FMA2) {
       // two independent fused updates: every operand is loaded before either store
+      // (the plain variant is given the unpaired stream and does not carry this path)
       const T x1 = flip_sign(L.lds(f[1]), in.flags & 1), y1 = L.lds(f[2]), c1 = L.lds(f[3]), g1 = L.lds(f[4]);
       const T x2 = flip_sign(L.lds(f[6]), (in.flags >> 1) & 1), y2 = L.lds(f[7]), c2 = L.lds(in.pad3),
               g2 = L.lds(in.pad4);
