@@ -258,8 +258,9 @@ __device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w
 // by the owner of element 0, and a warp barrier after every instruction publishes
 // the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
 // cost while G times more warps cover the lanes.
-template <typename T, bool SHARED, bool STAGED>
+template <typename T, bool SHARED, bool STAGED, bool BLOCK>
 __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(ReplayArgs a) {
+  static_assert(!BLOCK || SHARED, "a block-cooperative lane is an element-split group");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
@@ -296,8 +297,10 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
   const bool writer = live && grank == 0;
   // element-split groups publish each instruction's writes: a warp barrier when the
   // group lies within a warp, a block barrier when one lane spans the whole block
+  // (BLOCK: one lane per block, G = the block; a separate variant, so that the
+  // in-warp groups do not carry the block-mode paths)
   const bool sync_each = SHARED && G > 1;
-  const bool sync_block = SHARED && G > 32;
+  const bool sync_block = BLOCK;
   auto group_sync = [&]() {
     if (sync_block) __syncthreads();
     else __syncwarp();
@@ -802,7 +805,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
   }
 }
 
-template <typename T, bool SHARED, bool STAGED>
+template <typename T, bool SHARED, bool STAGED, bool BLOCK>
 cudaError_t launch_v(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
   static int configured_dev = -1;
   static size_t configured_smem = 0;
@@ -810,20 +813,25 @@ cudaError_t launch_v(const ReplayArgs& a, int blocks, int tpb, size_t smem, cuda
   cudaGetDevice(&dev);
   if (configured_dev != dev || smem > configured_smem) {
     cudaError_t e =
-        cudaFuncSetAttribute(k_replay<T, SHARED, STAGED>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(k_replay<T, SHARED, STAGED, BLOCK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     configured_dev = dev;
     configured_smem = smem;
   }
-  k_replay<T, SHARED, STAGED><<<blocks, tpb, smem, s>>>(a);
+  k_replay<T, SHARED, STAGED, BLOCK><<<blocks, tpb, smem, s>>>(a);
   return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t launch_t(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  if (a.shared_lane && (1 << a.log2g) > 32)  // one lane per block
+    return a.staged ? launch_v<T, true, true, true>(a, blocks, tpb, smem, s)
+                    : launch_v<T, true, false, true>(a, blocks, tpb, smem, s);
   if (a.shared_lane)
-    return a.staged ? launch_v<T, true, true>(a, blocks, tpb, smem, s) : launch_v<T, true, false>(a, blocks, tpb, smem, s);
-  return a.staged ? launch_v<T, false, true>(a, blocks, tpb, smem, s) : launch_v<T, false, false>(a, blocks, tpb, smem, s);
+    return a.staged ? launch_v<T, true, true, false>(a, blocks, tpb, smem, s)
+                    : launch_v<T, true, false, false>(a, blocks, tpb, smem, s);
+  return a.staged ? launch_v<T, false, true, false>(a, blocks, tpb, smem, s)
+                  : launch_v<T, false, false, false>(a, blocks, tpb, smem, s);
 }
 
 }  // namespace
