@@ -274,7 +274,7 @@ def main():
     esz = np.dtype(npdt).itemsize
     for tp, w in zip(tapes, progs):
         c = tp.cost()
-        work += (c["work_fwd"] + c["work_rev"]) * w.B
+        work += (c["work_fwd"] + c["work_rev"]) * w.B + c["work_shared"]
         alg_bytes += (2 * c["save_elems"] + 2 * w.P + 1) * esz * w.B + esz * w.obs.size
 
     # independent programs run on several streams so their kernels co-reside on the SMs

@@ -187,6 +187,14 @@ ndvm_status ndvm_tape_cost(const ndvm_tape* tape, double* work_fwd, double* work
                            int32_t* flags);
 
 /*
+ * ndvm_tape_shared_work -- FP64 work (DFMA-equivalents) per value-and-gradient call
+ * that does not scale with the lanes: the shared per-point values of data-axis regions
+ * (section 3.5: values that depend on the data point but on no parameter are the same
+ * on every lane, so they are computed once per call).  0 when there are none.
+ */
+ndvm_status ndvm_tape_shared_work(const ndvm_tape* tape, double* work_per_call);
+
+/*
  * ndvm_measure_fp64_peak -- measure the device's FP64 fused multiply-add rate
  * (flop/s, two per FMA) with a dependent-chain microbenchmark on all SMs; the
  * roofline denominator for the replay, which is bound by FP64 issue.  Synchronous.

@@ -65,6 +65,7 @@ def load(build_if_missing: bool = True):
             "ndvm_value_and_grad_host": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_value_and_grad_noalloc": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_value_and_grad_host_async": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
+            "ndvm_tape_shared_work": (ctypes.c_int, [P, ctypes.POINTER(ctypes.c_double)]),
             "ndvm_check_device": (ctypes.c_int, [P]),
             "ndvm_launch_count": (ctypes.c_ulonglong, []),
             "ndvm_measure_fp64_peak": (ctypes.c_int, [ctypes.POINTER(ctypes.c_double), P]),
@@ -112,8 +113,10 @@ class Tape:
         se, fl = ctypes.c_int64(), ctypes.c_int32()
         _check(lib.ndvm_tape_cost(self.handle, ctypes.byref(wf), ctypes.byref(wr), ctypes.byref(se),
                                   ctypes.byref(fl)))
+        ws = ctypes.c_double()
+        _check(lib.ndvm_tape_shared_work(self.handle, ctypes.byref(ws)))
         return {"work_fwd": wf.value, "work_rev": wr.value, "save_elems": se.value,
-                "has_regions": bool(fl.value & 1), "spill": bool(fl.value & 2)}
+                "has_regions": bool(fl.value & 1), "spill": bool(fl.value & 2), "work_shared": ws.value}
 
     def serialize(self) -> bytes:
         lib = load()

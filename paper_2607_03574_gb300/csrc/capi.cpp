@@ -33,6 +33,7 @@ ndvm_status cuda_fail(cudaError_t e, const char* where) {
 }
 
 struct DevPlan {
+  std::vector<DevPlan> derive;  // derive plans of the shared per-point values
   DInst* code = nullptr;
   DInst* code_paired = nullptr;  // the paired stream (staged and element-split variants), or null
   int32_t* args = nullptr;
@@ -64,6 +65,7 @@ struct ndvm_tape {
 namespace {
 
 void free_plan(DevPlan& p) {
+  for (DevPlan& d : p.derive) free_plan(d);
   cudaFree(p.code); cudaFree(p.code_paired); cudaFree(p.args); cudaFree(p.consts_d); cudaFree(p.consts_f);
   p = DevPlan{};
 }
@@ -87,6 +89,11 @@ ndvm_status upload_plan(const Tape& t, const Plan& p, DevPlan& d) {
     if ((e = cudaMalloc(&d.code_paired, sizeof(DInst) * (p.code_paired.size() + 1))) != cudaSuccess) return cuda_fail(e, "cudaMalloc");
     if ((e = cudaMemcpy(d.code_paired, p.code_paired.data(), sizeof(DInst) * p.code_paired.size(), cudaMemcpyHostToDevice)) != cudaSuccess)
       return cuda_fail(e, "cudaMemcpy");
+  }
+  d.derive.resize(p.derive.size());
+  for (size_t k = 0; k < p.derive.size(); k++) {
+    ndvm_status s = upload_plan(t, p.derive[k], d.derive[k]);
+    if (s != NDVM_OK) return s;
   }
   if ((e = cudaMemcpy(d.args, args.data(), sizeof(int32_t) * args.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
   if ((e = cudaMemcpy(d.consts_d, c.data(), sizeof(double) * c.size(), cudaMemcpyHostToDevice)) != cudaSuccess) return cuda_fail(e, "cudaMemcpy");
@@ -233,6 +240,59 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
   return s;
 }
 
+// bytes of the extended observations (a copy of the observations the program reads,
+// then the regions' blocks of shared per-point values), rounded up to 256; 0 without
+size_t derived_bytes(const Plan& p, size_t elem) {
+  if (p.derive.empty()) return 0;
+  return ((size_t)(p.n_obs_min + p.derived_elems) * elem + 255) / 256 * 256;
+}
+
+// Fill the extended observations at `ext`: copy obs[0 .. n_obs_min), then run the derive
+// plans, one lane per point of each region, each lane's parameters being its point's
+// observation record (params = obs + base, P = stride).
+ndvm_status run_derive(const Plan& p, const DevPlan& dp, ndvm_dtype dtype, const void* obs, void* ext, int* err,
+                       void* stream) {
+  const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  cudaError_t e = cudaMemcpyAsync(ext, obs, (size_t)p.n_obs_min * elem, cudaMemcpyDeviceToDevice, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "copy observations");
+  for (size_t k = 0; k < p.derive.size(); k++) {
+    const Plan& q = p.derive[k];
+    const DeriveInfo& di = p.derive_info[k];
+    const DevPlan& dq = dp.derive[k];
+    if (di.n_points <= 0) continue;
+    const Shape sh = launch_shape(q, elem, di.n_points);
+    ReplayArgs a;
+    a.code = dq.code;
+    a.n_code = (int)q.code.size();
+    a.args = dq.args;
+    a.consts = dtype == NDVM_F32 ? (const void*)dq.consts_f : (const void*)dq.consts_d;
+    a.obs = obs;
+    a.params = static_cast<const char*>(obs) + (size_t)di.base * elem;
+    a.loss = nullptr;
+    a.grad = nullptr;
+    a.save = static_cast<char*>(ext) + (size_t)(p.n_obs_min + di.offset) * elem;
+    a.save_ld = di.n_points;
+    a.P = (int)di.stride;
+    a.log2g = sh.log2g;
+    a.shared_lane = sh.shared;
+    a.sstride = sh.sstride;
+    a.staged = sh.staged;
+    a.stage_off = sh.stage_off;
+    a.err = err;
+    a.lane0 = 0;
+    a.lane_end = di.n_points;
+    const int64_t lanes_per_block = sh.tpb >> sh.log2g;
+    const int64_t blocks = (di.n_points + lanes_per_block - 1) / lanes_per_block;
+    {
+      std::lock_guard<std::mutex> lk(g_launch_mu);
+      e = launch_replay(a, dtype == NDVM_F32, (int)blocks, sh.tpb, sh.smem, (cudaStream_t)stream);
+      g_launches++;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "derive launch");
+  }
+  return NDVM_OK;
+}
+
 ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
                 int64_t n_obs, void* loss, void* gradp, void* ws, size_t ws_bytes, void* stream) {
   if (!t) return fail(NDVM_E_INVALID_ARG, "null tape");
@@ -252,6 +312,12 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   const size_t smem = sh.smem;
   if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs " + std::to_string(p.n_slots) + " slots per lane, more than shared memory holds");
   const int lanes_per_block = tpb >> log2g;
+  // the workspace holds the shared per-point values first, then the per-lane saves
+  const size_t der_bytes = grad ? derived_bytes(p, elem) : 0;
+  if (der_bytes > 0 && (!ws || ws_bytes < der_bytes))
+    return fail(NDVM_E_INVALID_ARG, "this tape needs a workspace of at least " + std::to_string(der_bytes) + " bytes");
+  void* lane_ws = der_bytes > 0 ? static_cast<char*>(ws) + der_bytes : ws;
+  if (der_bytes > 0) ws_bytes -= der_bytes;
   int64_t chunk = B;
   if (grad && p.n_save > 0) {
     const size_t per_lane = (size_t)p.n_save * elem;
@@ -269,6 +335,7 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   ndvm_status s = device_cache(t, &dc);
   if (s != NDVM_OK) return s;
   const DevPlan& dp = grad ? dc->grad : dc->value;
+  if (der_bytes > 0 && (s = run_derive(p, dp, dtype, obs, ws, dc->err, stream)) != NDVM_OK) return s;
   ReplayArgs a;
   // the staged and element-split variants run the paired stream; the plain one does not
   // carry the paired instruction (it would cost its register budget)
@@ -277,11 +344,11 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   a.n_code = (int)(paired ? p.code_paired.size() : p.code.size());
   a.args = dp.args;
   a.consts = dtype == NDVM_F32 ? (const void*)dp.consts_f : (const void*)dp.consts_d;
-  a.obs = obs;
+  a.obs = der_bytes > 0 ? ws : obs;  // the extended observations when the tape has shared values
   a.params = params;
   a.loss = loss;
   a.grad = gradp;
-  a.save = ws;
+  a.save = lane_ws;
   a.save_ld = chunk;
   a.P = p.n_params;
   a.log2g = log2g;
@@ -374,6 +441,14 @@ ndvm_status ndvm_tape_cost(const ndvm_tape* t, double* work_fwd, double* work_re
   return NDVM_OK;
 }
 
+ndvm_status ndvm_tape_shared_work(const ndvm_tape* t, double* work_per_call) {
+  if (!t || !work_per_call) return fail(NDVM_E_INVALID_ARG, "null argument");
+  double w = 0;
+  for (const DeriveInfo& di : t->grad_plan.derive_info) w += di.work * (double)di.n_points;
+  *work_per_call = w;
+  return NDVM_OK;
+}
+
 ndvm_status ndvm_tape_serialize(const ndvm_tape* t, void* buf, size_t cap, size_t* len) {
   if (!t || !len) return fail(NDVM_E_INVALID_ARG, "null argument");
   std::vector<uint8_t> s = t->tape.serialize();
@@ -402,7 +477,7 @@ void ndvm_tape_free(ndvm_tape* t) {
 size_t ndvm_workspace_bytes(const ndvm_tape* t, int64_t B, ndvm_dtype dtype) {
   if (!t || B <= 0) return 0;
   size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
-  return (size_t)t->grad_plan.n_save * elem * (size_t)B;
+  return derived_bytes(t->grad_plan, elem) + (size_t)t->grad_plan.n_save * elem * (size_t)B;
 }
 
 ndvm_status ndvm_forward(const ndvm_tape* tape, ndvm_dtype dtype, int64_t B, const void* params, const void* obs,
@@ -525,15 +600,21 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   const size_t smem = sh.smem;
   if (smem > kSmemLimit) return fail(NDVM_E_UNSUPPORTED, "tape needs more slots per lane than shared memory holds");
   const int lanes_per_block = tpb >> log2g;
+  // the scratch holds the shared per-point values first, then the per-lane saves
+  const size_t der_bytes = derived_bytes(p, elem);
+  const size_t lane_scratch = der_bytes <= kNoAllocScratchBytes ? kNoAllocScratchBytes - der_bytes : 0;
   int64_t chunk = B;
+  if (der_bytes > kNoAllocScratchBytes)
+    return fail(NDVM_E_INVALID_ARG, "this tape's extended observations need " + std::to_string(der_bytes) +
+                                        " bytes; the fixed scratch holds " + std::to_string(kNoAllocScratchBytes) + " bytes");
   if (p.n_save > 0) {
     const size_t per_lane = (size_t)p.n_save * elem;
     const size_t per_block = per_lane * lanes_per_block;
-    if (per_block > kNoAllocScratchBytes)
+    if (per_block > lane_scratch)
       return fail(NDVM_E_INVALID_ARG, "this tape needs " + std::to_string(per_block) + " bytes of workspace per block of " +
                                           std::to_string(lanes_per_block) + " lanes; the fixed scratch holds " +
                                           std::to_string(kNoAllocScratchBytes) + " bytes");
-    int64_t fit = (int64_t)(kNoAllocScratchBytes / per_lane);
+    int64_t fit = (int64_t)(lane_scratch / per_lane);
     if (fit < B) chunk = fit - fit % lanes_per_block;
   }
   DevCache* dc = nullptr;
@@ -551,17 +632,21 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   void* scratch = nullptr;
   cudaError_t e = noalloc_scratch(&scratch);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress");
+  if (der_bytes > 0) {
+    ndvm_status s = run_derive(p, dc->grad, dtype, obs, scratch, dc->err, stream);
+    if (s != NDVM_OK) return s;
+  }
   ReplayArgs a;
   const bool paired = (sh.staged || sh.shared) && dc->grad.code_paired != nullptr;
   a.code = paired ? dc->grad.code_paired : dc->grad.code;
   a.n_code = (int)(paired ? p.code_paired.size() : p.code.size());
   a.args = dc->grad.args;
   a.consts = dtype == NDVM_F32 ? (const void*)dc->grad.consts_f : (const void*)dc->grad.consts_d;
-  a.obs = obs;
+  a.obs = der_bytes > 0 ? scratch : obs;
   a.params = params;
   a.loss = loss;
   a.grad = grad;
-  a.save = scratch;
+  a.save = static_cast<char*>(scratch) + der_bytes;
   a.save_ld = chunk;
   a.P = p.n_params;
   a.log2g = log2g;

@@ -15,6 +15,7 @@
 #include <climits>
 #include <cstdlib>
 #include <cstring>
+#include <functional>
 #include <map>
 #include <set>
 
@@ -29,6 +30,12 @@ namespace {
 // NDVM_PREFETCH=0 disables the reverse sweep's workspace prefetch (a tuning knob).
 bool prefetch_enabled() {
   const char* e = std::getenv("NDVM_PREFETCH");
+  return !(e && e[0] == '0');
+}
+
+// NDVM_DERIVE=0 computes the shared per-point values on every lane instead.
+bool derive_enabled() {
+  const char* e = std::getenv("NDVM_DERIVE");
   return !(e && e[0] == '0');
 }
 
@@ -118,6 +125,17 @@ class Planner {
   std::vector<uint8_t> active_, region_body_;
   std::vector<char> need_val_, need_aux_;
   std::vector<int> twin_inv_;  // DET/LOGDET node -> an INV node of the same matrix (or -1)
+  // shared per-point values: pdep_ = depends on a parameter; derived_ = a region body
+  // node computed by a derive plan instead; der_col_ = its column when the replay reads it
+  std::vector<char> pdep_, derived_;
+  std::vector<int> der_col_;
+  std::vector<int> der_of_;       // DSUM node -> index of its derive plan (or -1)
+  int emit_r_ = -1;               // DSUM node whose body is being emitted (forward or reverse)
+  std::vector<DeriveInfo> der_info_;
+  std::vector<int> der_region_;   // DSUM node of each derive plan
+  int64_t der_elems_ = 0;
+  void plan_derived();
+  Plan build_derive(int r, const DeriveInfo& info) const;
   std::vector<int> val_vr_, aux_vr_, adj_vr_;
   std::vector<int64_t> save_, aux_save_;
   std::vector<VR> vrs_;
@@ -285,6 +303,13 @@ void Planner::analyze() {
 
 PRef Planner::ref(int v) {
   const Node& n = T.nodes[v];
+  if (emit_r_ >= 0 && der_of_[emit_r_] >= 0) {
+    // a region with shared per-point values reads its point's observations and derived
+    // values from the region's block of the extended observations, column-major
+    const DeriveInfo& di = der_info_[der_of_[emit_r_]];
+    if (n.op == OP_DOBS) return kref(RK_DOBS, (int32_t)(n.imm * di.n_points));
+    if (der_col_[v] >= 0) return kref(RK_DOBS, (int32_t)((di.obs_cols + der_col_[v]) * di.n_points));
+  }
   switch (n.op) {
     case OP_CONST: return kref(RK_CONST, n.imm);
     case OP_PARAM: return kref(RK_PARAM, n.imm);
@@ -562,12 +587,18 @@ void Planner::emit_region(int v) {
   PInst z; z.d.op = D_ZERO; z.f[0] = R(slotref(block)); z.f[1] = I(1 + (int)ins.size());
   emit(z);
   PInst lp; lp.d.op = D_LOOP; lp.f[0] = I(n.imm); lp.f[1] = I(stride); lp.f[2] = I(base);
+  if (der_of_[v] >= 0) {  // the region's block of the extended observations
+    lp.f[1] = I(1);
+    lp.f[2] = I((int32_t)(T.n_obs_min + der_info_[der_of_[v]].offset));
+  }
+  emit_r_ = v;
   int loop_pc = emit(lp);
   mult_ = (double)n.imm;
   work_fwd_ += mult_;  // accumulation of the body value
   for (int u = b0; u < b1; u++) {
     if (!body_value(u)) continue;
     if (T.nodes[u].op == OP_DSUM) unsupported("nested data-sum");
+    if (!derived_.empty() && derived_[u]) continue;  // a shared per-point value
     emit_forward(u);
   }
   PInst acc; acc.d.op = D_ACC; acc.f[0] = R(slotref(block, 0)); acc.f[1] = R(ref(res));
@@ -601,6 +632,198 @@ void Planner::emit_region(int v) {
   code_[loop_pc].f[3] = I(end_pc);
   PInst gr; gr.d.op = D_GREDUCE; gr.f[0] = R(slotref(block)); gr.f[1] = I(1 + (int)ins.size());
   emit(gr);
+  emit_r_ = -1;
+}
+
+// Shared per-point values.  Inside a data-axis region, a body node that depends on the
+// data point but on no parameter has the same value on every lane.  When every such
+// node of a region is a scalar primitive, they move to a derive plan (run once per call,
+// one lane per point); the replay reads the ones that parameter-dependent nodes (or the
+// region's sum) use from the derived buffer.  The values are the same IEEE results in
+// the same order, computed once instead of once per lane.
+void Planner::plan_derived() {
+  pdep_.assign(N, 0);
+  for (int v = 0; v < N; v++) {
+    if (T.nodes[v].op == OP_PARAM) { pdep_[v] = 1; continue; }
+    for (int x : inputs(v)) if (x >= 0 && x < v && pdep_[x]) { pdep_[v] = 1; break; }
+  }
+  derived_.assign(N, 0);
+  der_col_.assign(N, -1);
+  der_of_.assign(N, -1);
+  if (!grad_ || !derive_enabled()) return;
+  auto scalar_prim = [&](int u) {
+    const Node& m = T.nodes[u];
+    if (m.rows != 1 || m.cols != 1) return false;
+    switch (m.op) {
+      case OP_ADD: case OP_SUB: case OP_MUL: case OP_DIV: case OP_POW: case OP_NEG: case OP_EXP: case OP_LOG:
+      case OP_SIN: case OP_COS: case OP_TANH: case OP_SQRT: case OP_ABS: case OP_POWI: case OP_LT: case OP_LE:
+      case OP_GT: case OP_GE: case OP_EQ: case OP_SELECT:
+        return true;
+      default:
+        return false;
+    }
+  };
+  for (int r = 0; r < N; r++) {
+    const Node& n = T.nodes[r];
+    if (n.op != OP_DSUM) continue;
+    std::vector<int> cand;
+    bool ok = true;
+    for (int u = n.a; u < n.b && ok; u++) {
+      if (!region_body_[u] || is_leaf(u) || pdep_[u]) continue;
+      if (!scalar_prim(u)) ok = false;
+      else cand.push_back(u);
+    }
+    if (!ok || cand.empty()) continue;
+    // inputs of the candidates that are neither leaves nor candidates are lane-level
+    // values without parameters (constant subexpressions hoisted out of the body): the
+    // derive plan recomputes them, so they too must be scalar primitives
+    std::vector<char> incand(N, 0), seen(N, 0);
+    for (int u : cand) incand[u] = 1;
+    std::vector<int> stack;
+    for (int u : cand)
+      for (int x : inputs(u)) stack.push_back(x);
+    while (!stack.empty() && ok) {
+      const int x = stack.back();
+      stack.pop_back();
+      if (x < 0 || seen[x] || incand[x] || is_leaf(x)) continue;
+      seen[x] = 1;
+      if (pdep_[x] || !scalar_prim(x)) { ok = false; break; }
+      for (int y : inputs(x)) stack.push_back(y);
+    }
+    if (!ok) continue;
+    for (int u : cand) derived_[u] = 1;
+    // columns: derived values that the replay reads
+    std::vector<char> used(N, 0);
+    for (int w = n.a; w < n.b; w++)
+      if (region_body_[w] && !is_leaf(w) && !derived_[w])
+        for (int x : inputs(w)) if (x >= 0 && derived_[x]) used[x] = 1;
+    if (derived_[n.c]) used[n.c] = 1;
+    DeriveInfo info;
+    info.n_points = n.imm;
+    info.stride = T.args[n.imm2];
+    info.base = T.args[n.imm2 + 1];
+    info.offset = der_elems_;
+    // observation columns the region reads (copied into its block)
+    int maxk = -1;
+    for (int w = n.a; w < n.b; w++) {
+      if (!region_body_[w] || is_leaf(w)) continue;
+      for (int x : inputs(w))
+        if (x >= 0 && T.nodes[x].op == OP_DOBS) maxk = std::max(maxk, T.nodes[x].imm);
+    }
+    if (T.nodes[n.c].op == OP_DOBS) maxk = std::max(maxk, T.nodes[n.c].imm);
+    info.obs_cols = maxk + 1;
+    int ncols = 0;
+    for (int u : cand) {
+      if (used[u]) der_col_[u] = ncols++;
+      const Node& m = T.nodes[u];
+      info.work += cost::fwd(m.op, 1, 1, m.imm, 1, false);
+    }
+    info.n_cols = info.obs_cols + ncols;
+    if ((int64_t)info.n_cols * info.n_points >= ((int64_t)1 << 27) ||
+        T.n_obs_min + der_elems_ + (int64_t)info.n_cols * info.n_points >= ((int64_t)1 << 30)) {
+      for (int u : cand) { derived_[u] = 0; der_col_[u] = -1; }  // outside the index range: keep per lane
+      continue;
+    }
+    der_of_[r] = (int)der_info_.size();
+    der_elems_ += info.n_points * info.n_cols;
+    der_info_.push_back(info);
+    der_region_.push_back(r);
+  }
+}
+
+// The derive plan of region r: one slot per value, leaves loaded first, the region's
+// derived nodes in tape order, each read value stored to its column (lanes = points).
+Plan Planner::build_derive(int r, const DeriveInfo& info) const {
+  const Node& n = T.nodes[r];
+  Plan pl;
+  // the point's observation record is the lane's parameter vector (params = obs + base,
+  // P = stride), so observation column k of point d is parameter k of lane d
+  pl.n_params = info.obs_cols;
+  for (int u = n.a; u < n.b; u++)
+    if (derived_[u])
+      for (int x : inputs(u))
+        if (x >= 0 && T.nodes[x].op == OP_DOBS) pl.n_params = std::max(pl.n_params, T.nodes[x].imm + 1);
+  pl.n_obs_min = T.n_obs_min;
+  pl.n_save = info.n_cols;
+  pl.extra_consts = {1.0, -0.0};
+  const int32_t k_one = (int32_t)T.consts.size(), k_mzero = k_one + 1;
+  std::vector<int> slot(N, -1);
+  int next = 0;
+  auto load = [&](uint32_t kind, int32_t idx) {
+    DInst d;
+    d.op = D_LOAD;
+    d.f[0] = mkref(RK_SLOT, next);
+    d.f[1] = mkref(kind, idx);
+    pl.code.push_back(d);
+    return next++;
+  };
+  auto leaf_slot = [&](int x) {
+    if (slot[x] >= 0) return slot[x];
+    const Node& m = T.nodes[x];
+    const uint32_t kind = m.op == OP_CONST ? RK_CONST : m.op == OP_OBS ? RK_OBS : RK_PARAM;
+    return slot[x] = load(kind, m.imm);
+  };
+  // copies of the observation columns into the block (exact: x * 1 + (-0) = x)
+  const int one = load(RK_CONST, k_one), mzero = load(RK_CONST, k_mzero);
+  for (int k = 0; k < info.obs_cols; k++) {
+    const int xk = load(RK_PARAM, k);
+    DInst d;
+    d.op = D_FMA;
+    d.f[0] = mkref(RK_SLOT, next++);
+    d.f[1] = mkref(RK_SLOT, xk);
+    d.f[2] = mkref(RK_SLOT, one);
+    d.f[3] = mkref(RK_SLOT, mzero);
+    d.f[4] = mkref(RK_SLOT, one);
+    d.f[5] = k;
+    pl.code.push_back(d);
+  }
+  // a value of the plan: a leaf is loaded, a derived node was computed in tape order, and
+  // a hoisted parameter-free lane-level node is computed on first use
+  std::function<int32_t(int)> sref;
+  auto emit_node = [&](int u, int32_t save_col) {
+    const Node& m = T.nodes[u];
+    int32_t ins[3] = {-1, -1, -1};
+    if (m.op == OP_SELECT) { ins[0] = sref(m.a); ins[1] = sref(m.b); ins[2] = sref(m.c); }
+    else { if (m.a >= 0) ins[0] = sref(m.a); if (m.b >= 0) ins[1] = sref(m.b); }
+    DInst d;
+    d.f[3] = save_col;
+    switch (m.op) {
+      case OP_ADD: d.op = D_ADD; break;
+      case OP_SUB: d.op = D_SUB; break;
+      case OP_MUL: d.op = D_MUL; break;
+      case OP_DIV: d.op = D_DIV; break;
+      case OP_POW: d.op = D_POW; break;
+      case OP_NEG: d.op = D_NEG; break;
+      case OP_EXP: d.op = D_EXP; break;
+      case OP_LOG: d.op = D_LOG; break;
+      case OP_SIN: d.op = D_SIN; break;
+      case OP_COS: d.op = D_COS; break;
+      case OP_TANH: d.op = D_TANH; break;
+      case OP_SQRT: d.op = D_SQRT; break;
+      case OP_ABS: d.op = D_ABS; break;
+      case OP_POWI: d.op = D_POWI; d.f[7] = m.imm; break;
+      case OP_SELECT: d.op = D_SELECT; break;
+      default:
+        d.op = D_CMP;
+        d.k = m.op == OP_LT ? 0 : m.op == OP_LE ? 1 : m.op == OP_GT ? 2 : m.op == OP_GE ? 3 : 4;
+        break;
+    }
+    if (m.op == OP_SELECT) { d.f[1] = ins[0]; d.f[2] = ins[1]; d.f[4] = ins[2]; }
+    else { d.f[1] = ins[0]; d.f[2] = ins[1]; }
+    d.f[0] = mkref(RK_SLOT, next);
+    pl.code.push_back(d);
+    slot[u] = next++;
+  };
+  sref = [&](int x) -> int32_t {
+    if (is_leaf(x)) return mkref(RK_SLOT, leaf_slot(x));
+    if (slot[x] < 0) emit_node(x, -1);  // a hoisted constant subexpression
+    return mkref(RK_SLOT, slot[x]);
+  };
+  for (int u = n.a; u < n.b; u++)
+    if (derived_[u]) emit_node(u, der_col_[u] >= 0 ? info.obs_cols + der_col_[u] : -1);
+  pl.n_slots = next;
+  pl.work_fwd = info.work;
+  return pl;
 }
 
 // The constant pool index holding exactly the bits of v (appended when absent).
@@ -897,6 +1120,7 @@ Plan Planner::build() {
   if (one_const_ < 0) { extra_consts_.push_back(1.0); one_const_ = (int)T.consts.size(); }
   if (T.loss < 0 || T.loss >= (int)T.nodes.size()) unsupported("tape has no loss");
   analyze();
+  plan_derived();
   Plan pl;
   pl.grad = grad_;
   pl.spill = spill_;
@@ -943,6 +1167,8 @@ Plan Planner::build() {
   pl.n_params = T.n_params;
   pl.n_obs_min = T.n_obs_min;
   for (const Node& nd : T.nodes) if (nd.op == OP_DOBS && nd.imm > pl.max_dobs) pl.max_dobs = nd.imm;
+  for (const DeriveInfo& di : der_info_)  // column-major block reads: up to the last column's start
+    pl.max_dobs = std::max<int32_t>(pl.max_dobs, (int32_t)((di.n_cols - 1) * di.n_points));
   for (const PInst& p : code_) {
     DInst d = p.d;
     for (int k = 0; k < 8; k++) d.f[k] = encode(p.f[k]);
@@ -954,6 +1180,9 @@ Plan Planner::build() {
     if (d.op == D_MATMUL || d.op == D_MADD || d.op == D_MSUB || d.op == D_MSCALE || d.op == D_INV ||
         ((d.op == D_DET || d.op == D_LOGDET) && d.r > 1) || (d.op == D_GATHER && d.f[2] > 1))
       pl.has_matrix = true;
+  for (size_t k = 0; k < der_info_.size(); k++) pl.derive.push_back(build_derive(der_region_[k], der_info_[k]));
+  pl.derive_info = der_info_;
+  pl.derived_elems = der_elems_;
   pl.extra_consts = extra_consts_;
   pl.work_fwd = work_fwd_;
   pl.work_rev = work_rev_;
@@ -992,6 +1221,9 @@ Plan make_plan(const Tape& t, bool grad, int force_mode) {
 bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_consts, std::string& why);
 
 bool validate_plan(const Plan& p, size_t n_consts, std::string& why) {
+  if (p.derive.size() != p.derive_info.size()) { why = "derive plans"; return false; }
+  for (const Plan& d : p.derive)
+    if (!d.derive.empty() || !validate_code(d, d.code, n_consts, why)) return false;
   return validate_code(p, p.code, n_consts, why) &&
          (p.code_paired.empty() || validate_code(p, p.code_paired, n_consts, why));
 }
@@ -1068,6 +1300,10 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
       case D_LOOP:
         ok = open_loop < 0 && f[3] > (int)pc && f[3] < (int)code.size() && code[f[3]].op == D_ENDLOOP &&
              f[0] >= 0 && f[1] >= 0 && f[2] >= 0;
+        // a region reading a block of the extended observations stays inside it
+        for (const DeriveInfo& di : p.derive_info)
+          if (ok && f[2] == p.n_obs_min + di.offset && f[1] == 1)
+            ok = f[0] == di.n_points && di.offset + di.n_points * di.n_cols <= p.derived_elems;
         open_loop = (int)pc;
         break;
       case D_ENDLOOP: ok = f[0] == open_loop && code[f[0]].f[3] == (int)pc; open_loop = -1; break;
@@ -1132,8 +1368,9 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
         break;
       default: why = "bad opcode"; return false;
     }
+    const bool forward_scalar = (d.op >= D_ADD && d.op <= D_SELECT) || d.op == D_ACC;
     for (int fld = 0; ok && fld < 8; fld++)
-      if (slot_operand(d.op, fld) && f[fld] != -1 && ref_kind(f[fld]) != RK_SLOT) ok = false;
+      if (slot_operand(d.op, fld) && (f[fld] == -1 ? forward_scalar : ref_kind(f[fld]) != RK_SLOT)) ok = false;
     if (!ok) { why = "operand out of range at instruction " + std::to_string(pc) + " (op " + std::to_string(d.op) + ")"; return false; }
   }
   if (open_loop >= 0) { why = "unterminated loop"; return false; }

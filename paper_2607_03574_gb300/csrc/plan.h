@@ -109,6 +109,23 @@ struct alignas(16) DInst {
 };
 static_assert(sizeof(DInst) == 48, "DInst layout");
 
+// Shared per-point values of a data-axis region.  The body nodes that depend on the data
+// point but on no parameter are the same on every lane, so a derive plan computes them
+// once per call (one lane per point) into an extended observation buffer:
+//   [ obs[0 .. n_obs_min) | region blocks ],
+// where region r's block, at n_obs_min + offset, holds columns [col][point] of N values:
+// first copies of the point's observation columns 0 .. obs_cols-1, then the derived
+// values.  The replay's loop over the region then reads column c of point d as
+// observation (n_obs_min + offset) + c * N + d: base n_obs_min + offset, stride 1, and
+// DOBS index c * N.
+struct DeriveInfo {
+  int64_t n_points = 0, stride = 0, base = 0;  // the region's points: obs[base + d*stride + k]
+  int64_t offset = 0;                          // block offset after the copied observations
+  int32_t obs_cols = 0;                        // observation columns copied into the block
+  int32_t n_cols = 0;                          // all columns of the block
+  double work = 0;                             // DFMA-equivalents per point
+};
+
 struct Plan {
   bool grad = false;          // has a reverse sweep
   bool spill = false;         // reverse reads primals from the HBM workspace
@@ -128,6 +145,12 @@ struct Plan {
   // algorithmic cost per lane (for the roofline): DFMA-equivalents and saved bytes
   double work_fwd = 0, work_rev = 0;
   double n_ops_per_lane = 0;
+  // shared per-point values (gradient plans of data-axis tapes): one forward-only plan
+  // per region, whose lanes are the points (its parameters are the point's observation
+  // record: params = obs + base, P = stride); derived_elems = size of the region blocks
+  std::vector<Plan> derive;
+  std::vector<DeriveInfo> derive_info;
+  int64_t derived_elems = 0;
 };
 
 // Build the plan; throws BuildError on unsupported tapes.
