@@ -175,19 +175,24 @@ def cpu_sample_lanes(args, progs):
     return 2048 if args.config == 2 else progs[0].B
 
 
-def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = False):
-    """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program."""
+def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = False, min_seconds: float = 0.0):
+    """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program,
+    repeated until at least `min_seconds` have passed (small workloads)."""
     import oracle
     oracle.build()
     t0 = time.perf_counter()
     n = 0
-    for w in progs:
-        p = w.params[:lanes_per_prog]
-        if f32:
-            p = p.astype(np.float32).astype(np.float64)
-        oracle.run(w.program, p, w.obs, frontend=w.frontend, nthreads=nthreads, f32=f32)
-        n += len(p)
-    return n, time.perf_counter() - t0
+    while True:
+        for w in progs:
+            p = w.params[:lanes_per_prog]
+            if len(p) < 1024:  # small populations: tile the lanes so thread start-up does not dominate
+                p = np.resize(p, (1024, p.shape[1]))
+            if f32:
+                p = p.astype(np.float32).astype(np.float64)
+            oracle.run(w.program, p, w.obs, frontend=w.frontend, nthreads=nthreads, f32=f32)
+            n += len(p)
+        if time.perf_counter() - t0 >= min_seconds:
+            return n, time.perf_counter() - t0
 
 
 def run_reference(args):
@@ -200,13 +205,15 @@ def run_reference(args):
     f32 = args.dtype == "f32"
     for _ in range(args.warmup):
         oracle_sample_time(progs[:4], 2, cores, f32)
-    times, n = [], 0
-    for _ in range(args.steps):
-        n, dt = oracle_sample_time(progs, lanes, cores, f32)
-        times.append(dt)
-    ms = 1e3 * float(np.mean(times))
-    value = n / (ms * 1e-3)
-    sample = f"{lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals per step), whole data set"
+    ns, dts = [], []
+    for _ in range(args.steps):  # a step: the sample, repeated to at least a second for small workloads
+        n, dt = oracle_sample_time(progs, lanes, cores, f32, min_seconds=1.0)
+        ns.append(n)
+        dts.append(dt)
+    ms = 1e3 * float(np.mean(dts))
+    value = float(np.sum(ns)) / float(np.sum(dts))
+    sample = (f"{lanes} lanes of each of the {len(progs)} program(s), whole data set "
+              f"({int(np.mean(ns))} lane evals per step)")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -392,9 +399,10 @@ def main():
         f32 = args.dtype == "f32"
         lanes = cpu_sample_lanes(args, progs)
         oracle_sample_time(progs[:2], 2, cores, f32)
-        n, dt = oracle_sample_time(progs, lanes, cores, f32)
+        n, dt = oracle_sample_time(progs, lanes, cores, f32, min_seconds=2.0)
         cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{lanes} lanes of each of the {len(progs)} program(s) ({n} lane evals, {dt:.1f} s)"}
+               "sample": f"{lanes} lanes of each of the {len(progs)} program(s), repeated to {n} lane evals "
+                         f"({dt:.1f} s)"}
 
     if rank == 0:
         line = {
