@@ -362,3 +362,40 @@ def test_million_lanes_sampled(ndvm, oracle_mod, cuda):
     idx = np.array([0, 1, 12345, 524287, 524288, (1 << 20) - 1])
     ol, og, om = oracle_run(oracle_mod, w, idx)
     check(gl[idx], gg[idx], ol, og, om)
+
+
+TWO_REGION_PROG = """
+(model (params a b)
+  (+ (* 0.25 (data-sum 24 3 0 (let ((s (sin (* 2.0 (dobs 0)))) (c (exp (/ (dobs 1) 4.0))))
+                                (let ((r (- (* a s) (* b c) (dobs 2)))) (* r r)))))
+     (data-sum 10 2 72 (let ((q (log (+ 1.0 (* (dobs 1) (dobs 1))))))
+                         (* (+ a q) (- b (cos (dobs 0))))))
+     (data-sum 5 1 92 (* (dobs 0) (dobs 0)))))
+"""
+
+
+def test_shared_point_values_match_per_lane_values(ndvm, oracle_mod, cuda, monkeypatch):
+    """Values that depend on the data point but on no parameter are computed once per call
+    (three regions: shared values feeding parameter terms, a product of two shared values,
+    and a region that is shared as a whole). The replay with them equals, bit for bit,
+    the replay that recomputes them on every lane, and the oracle at 1e-12."""
+    import torch
+    rng = np.random.default_rng(21)
+    obs = rng.normal(size=97)
+    params = rng.normal(size=(70, 2))
+    w = W.Workload("regions", TWO_REGION_PROG, 0, params, obs, np.zeros(2))
+    shared = ndvm.trace_build(w.program)
+    monkeypatch.setenv("NDVM_DERIVE", "0")
+    per_lane = ndvm.trace_build(w.program)
+    monkeypatch.delenv("NDVM_DERIVE")
+    assert shared.cost()["work_shared"] > 0 and per_lane.cost()["work_shared"] == 0
+    assert shared.workspace_bytes(70) > 0
+    p = torch.tensor(params, device="cuda")
+    o = torch.tensor(obs, device="cuda")
+    l1, g1 = ndvm.value_and_grad(shared, p, o)
+    l2, g2 = ndvm.value_and_grad(per_lane, p, o)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(l1.cpu().numpy(), l2.cpu().numpy())
+    np.testing.assert_array_equal(g1.cpu().numpy(), g2.cpu().numpy())
+    ol, og, om = oracle_run(oracle_mod, w)
+    check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og, om)
