@@ -242,7 +242,7 @@ def main():
                          "every lane otherwise)")
     ap.add_argument("--lanes", type=int, default=0, help="lanes per program instead of the configuration's "
                                                          "(smaller cases for profiling)")
-    ap.add_argument("--streams", type=int, default=4, help="CUDA streams the programs are spread over")
+    ap.add_argument("--streams", type=int, default=16, help="CUDA streams the programs are spread over")
     ap.add_argument("--no-graph", dest="graph", action="store_false",
                     help="launch every step from the host instead of replaying a captured CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
