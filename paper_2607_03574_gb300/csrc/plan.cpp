@@ -33,6 +33,13 @@ bool prefetch_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_FETCHTRIM=0 keeps a fetch record, a commit and a wait in every window of the
+// reverse sweep, also where nothing is fetched (a tuning knob).
+bool fetch_trim_enabled() {
+  const char* e = std::getenv("NDVM_FETCHTRIM");
+  return !(e && e[0] == '0');
+}
+
 // NDVM_DERIVE=0 computes the shared per-point values on every lane instead.
 bool derive_enabled() {
   const char* e = std::getenv("NDVM_DERIVE");
@@ -45,13 +52,22 @@ bool pair_enabled() {
   return !(e && e[0] == '0');
 }
 
-// Two adjacent D_FMA records without saves, where the second neither reads the first's
-// result nor shares its destination, become one D_FMA2: one dispatch, both products in
-// flight together.  Runs on the encoded stream (physical slots): the kernel loads every
-// operand of the pair before it stores either result, so a second destination that
-// the first instruction reads is also safe.
+// NDVM_DEPPAIR=0 pairs independent fused instructions only (a tuning knob).
+bool dep_pair_enabled() {
+  const char* e = std::getenv("NDVM_DEPPAIR");
+  return !(e && e[0] == '0');
+}
+
+// Two adjacent D_FMA records without saves become one D_FMA2: one dispatch for both.
+// Runs on the encoded stream (physical slots).  The kernel loads every operand of the
+// pair before it stores either result, so a second destination that the first reads
+// is safe.  When the second reads the first's result (a chain, e.g. two contributions
+// accumulated into one adjoint), flags bit 2 tells the kernel to take that operand from
+// the first's result in a register; the two stores then run in order, so a shared
+// destination ends with the second's value.
 std::vector<DInst> pair_fma(const std::vector<DInst>& code) {
   const int n = (int)code.size();
+  const bool dep_ok = dep_pair_enabled();
   std::vector<DInst> out;
   out.reserve(n);
   std::vector<int> newpc(n, -1);
@@ -61,10 +77,10 @@ std::vector<DInst> pair_fma(const std::vector<DInst>& code) {
     if (pc + 1 < n && a.op == D_FMA && code[pc + 1].op == D_FMA && a.f[5] == -1 && code[pc + 1].f[5] == -1) {
       const DInst& b = code[pc + 1];
       const bool raw = b.f[1] == a.f[0] || b.f[2] == a.f[0] || b.f[3] == a.f[0] || b.f[4] == a.f[0];
-      if (!raw && b.f[0] != a.f[0]) {
+      if (raw ? dep_ok : b.f[0] != a.f[0]) {
         DInst q;
         q.op = D_FMA2;
-        q.flags = (uint8_t)((a.flags & 1) | ((b.flags & 1) << 1));
+        q.flags = (uint8_t)((a.flags & 1) | ((b.flags & 1) << 1) | (raw ? 4 : 0));
         for (int k = 0; k < 5; k++) q.f[k] = a.f[k];
         q.f[5] = b.f[0]; q.f[6] = b.f[1]; q.f[7] = b.f[2]; q.pad3 = b.f[3]; q.pad4 = b.f[4];
         out.push_back(q);
@@ -1014,9 +1030,25 @@ void Planner::prefetch_workspace() {
       pairs[k].push_back({fld, slot});
       fld = slot;
     }
-  // the fetch instructions of window k: kFetchPairs copies each, the last commits
-  auto fetches = [&](int k, bool wait, std::vector<PInst>& out) {
+  // The fetch instructions before window j issue the copies of window k = j + kFetchWindows
+  // (kFetchPairs per record) and commit them as one group, then wait for window j's
+  // group: at most n groups may stay pending, n = the groups committed after it (those
+  // of the windows j+1 .. j+kFetchWindows that fetch anything).  A window that fetches
+  // nothing commits no group, and one that reads nothing fetched waits for nothing; when
+  // both hold, no record is emitted (NDVM_FETCHTRIM=0 keeps one commit and a wait for
+  // kFetchWindows groups per window, empty ones included).
+  const bool trim = fetch_trim_enabled();
+  auto has = [&](int k) { return k >= 0 && k < nwin && !pairs[k].empty(); };
+  auto fetches = [&](int k, int j, std::vector<PInst>& out) {
     const int cnt = k < nwin ? (int)pairs[k].size() : 0;
+    bool wait = j >= 0;
+    int pending = kFetchWindows;
+    if (trim && wait) {
+      wait = has(j);
+      pending = 0;
+      for (int q = j + 1; q <= j + kFetchWindows; q++) pending += has(q) ? 1 : 0;
+    }
+    if (trim && cnt == 0 && !wait) return;
     int e = 0;
     do {
       PInst f;
@@ -1025,16 +1057,16 @@ void Planner::prefetch_workspace() {
       for (int q = 0; q < m; q++) { f.f[2 * q] = pairs[k][e + q].first; f.f[2 * q + 1] = pairs[k][e + q].second; }
       f.d.k = (uint8_t)m;
       e += m;
-      if (e >= cnt) f.d.flags = (uint8_t)(2 | (wait ? 1 : 0));
+      if (e >= cnt) f.d.flags = (uint8_t)(((cnt > 0 || !trim) ? 2 : 0) | (wait ? 1 | (pending << 2) : 0));
       out.push_back(f);
     } while (e < cnt);
   };
   std::vector<PInst> out(code_.begin(), code_.begin() + rev_begin_);
   std::vector<int> newpc(n, -1);
   for (int pc = 0; pc < rev_begin_; pc++) newpc[pc] = pc;
-  for (int k = 0; k < kFetchWindows; k++) fetches(k, false, out);  // prologue
+  for (int k = 0; k < kFetchWindows; k++) fetches(k, -1, out);  // prologue
   for (int k = 0; k < nwin; k++) {
-    fetches(k + kFetchWindows, true, out);
+    fetches(k + kFetchWindows, k, out);
     for (int pc = rev_begin_ + k * kFetchStride; pc < std::min(n, rev_begin_ + (k + 1) * kFetchStride); pc++) {
       newpc[pc] = (int)out.size();
       out.push_back(code_[pc]);
@@ -1361,7 +1393,7 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
         break;
       case B_GRAD: ok = ref_ok(f[0], 1, true) && f[1] >= 0 && f[1] < p.n_params; break;
       case D_FETCH:
-        ok = k <= kFetchPairs;
+        ok = k <= kFetchPairs && ((d.flags >> 2) & 7) <= kFetchWindows;
         for (int e = 0; ok && e < k; e++)
           ok = ref_kind(f[2 * e]) == RK_SAVE && ref_ok(f[2 * e], 1, false) && f[2 * e + 1] != -1 &&
                ref_ok(f[2 * e + 1], 1, true);

@@ -75,16 +75,17 @@ enum DOp : uint8_t {
   D_LOAD,           // slot f0 = ref f1 (a constant, parameter, observation or workspace value)
   D_FETCH,          // k = count <= kFetchPairs; pairs (f0 workspace ref, f1 slot), (f2, f3), ...:
                     // asynchronous copies into slots; flags bit1: then commit the copies issued
-                    // since the last commit as one group; bit0: then wait until at most
-                    // kFetchWindows groups are pending
+                    // since the last commit as one group; bit0: then wait until at most n groups
+                    // are pending, n = flags bits 2..4 (<= kFetchWindows)
   // ---- fused multiply-add form of the cheap scalar rules ----
   D_FMA,            // slot f0 = (is_zero(slot f4) ? slot f3 : fma(+-slot f1, slot f2, slot f3)), f5 save;
                     // flags bit0 negates the first factor.  f4 is the zero-skip test (an adjoint
                     // whose contribution vanishes when it is exactly zero; the slot holding 1.0
                     // when there is none)
-  D_FMA2,           // two independent D_FMA without saves in one record: (f0 dst, f1, f2, f3, f4 zero-skip)
+  D_FMA2,           // two D_FMA without saves in one record: (f0 dst, f1, f2, f3, f4 zero-skip)
                     // and (f5 dst, f6, f7, pad3, pad4 zero-skip); flags bit0 / bit1 negate the first
-                    // factor of the first / second
+                    // factor of the first / second; bit2: the second's operands that name f0 read
+                    // the first's result
   D_NOPS
 };
 

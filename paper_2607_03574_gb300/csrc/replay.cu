@@ -338,7 +338,9 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
     __syncthreads();
   }
   // non-staged streams: the record of the next instruction is loaded before the
-  // current one executes, so its latency overlaps the current instruction
+  // current one executes, so its latency overlaps the current instruction (the same
+  // look-ahead on the staged stream measured slower: it holds a second record in
+  // registers, and a shared-memory record is close at hand anyway)
   DInst nxt;
   if (!STAGED && a.n_code > 0) nxt = code[0];
   for (int pc = 0; pc < a.n_code; pc++) {
@@ -354,7 +356,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
     if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
 
     const int32_t* f = in.f;
-    if (in.op == 0 || in.op >= D_NOPS) {  // not an opcode: every thread stops together
+    if (BLOCK && (in.op == 0 || in.op >= D_NOPS)) {  // not an opcode: every thread stops together
       if (a.err && tid == 0) atomicExch(a.err, 1);
       return;
     }
@@ -384,12 +386,20 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       continue;
     }
     if ((SHARED || STAGED) && in.op == D_FMA2) {
-      // two independent fused updates: every operand is loaded before either store
+      // two fused updates in one record: every operand is loaded before either store;
+      // when the second reads the first's result (flags bit 2), the operands that name
+      // the first's destination take its value from the register instead
       // (the plain variant is given the unpaired stream and does not carry this path)
       const T x1 = flip_sign(L.lds(f[1]), in.flags & 1), y1 = L.lds(f[2]), c1 = L.lds(f[3]), g1 = L.lds(f[4]);
-      const T x2 = flip_sign(L.lds(f[6]), (in.flags >> 1) & 1), y2 = L.lds(f[7]), c2 = L.lds(in.pad3),
-              g2 = L.lds(in.pad4);
+      T x2 = L.lds(f[6]), y2 = L.lds(f[7]), c2 = L.lds(in.pad3), g2 = L.lds(in.pad4);
       const T z1 = is_zero(g1) ? c1 : fma(x1, y1, c1);
+      if (in.flags & 4) {
+        if (f[6] == f[0]) x2 = z1;
+        if (f[7] == f[0]) y2 = z1;
+        if (in.pad3 == f[0]) c2 = z1;
+        if (in.pad4 == f[0]) g2 = z1;
+      }
+      x2 = flip_sign(x2, (in.flags >> 1) & 1);
       const T z2 = is_zero(g2) ? c2 : fma(x2, y2, c2);
       L.st(f[0], 0, z1);
       L.st(f[5], 0, z2);
@@ -412,7 +422,15 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
             asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
         }
       if (in.flags & 2) asm volatile("cp.async.commit_group;\n" ::: "memory");
-      if (in.flags & 1) asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchWindows) : "memory");
+      if (in.flags & 1) {  // wait until at most n = flags bits 2..4 groups are pending
+        switch ((in.flags >> 2) & 7) {
+          case 0: asm volatile("cp.async.wait_group 0;\n" ::: "memory"); break;
+          case 1: asm volatile("cp.async.wait_group 1;\n" ::: "memory"); break;
+          case 2: asm volatile("cp.async.wait_group 2;\n" ::: "memory"); break;
+          case 3: asm volatile("cp.async.wait_group 3;\n" ::: "memory"); break;
+          default: asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchWindows) : "memory"); break;
+        }
+      }
       if (sync_each) group_sync();
       continue;
     }
@@ -796,7 +814,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       case B_GRAD:
         if (writer) grad[L.lane * L.P + f[1]] = f[0] == -1 ? (T)0 : L.sl(f[0], 0);
         break;
-      default:
+      default:  // not an opcode of this variant: every thread stops
         if (a.err) atomicExch(a.err, 1);
         if (sync_block) break;  // warp 0 alone may be here: keep the barrier count, stop nothing
         return;
