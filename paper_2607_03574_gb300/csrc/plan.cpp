@@ -98,6 +98,59 @@ std::vector<DInst> pair_fma(const std::vector<DInst>& code) {
   return out;
 }
 
+// NDVM_HOIST=0 keeps the seed of a data-axis body's reverse sweep inside the loop (a
+// tuning knob).
+bool hoist_enabled() {
+  const char* e = std::getenv("NDVM_HOIST");
+  return !(e && e[0] == '0');
+}
+
+// NDVM_MERGELOADS=0 keeps one record per observation load (a tuning knob).
+bool merge_loads_enabled() {
+  const char* e = std::getenv("NDVM_MERGELOADS");
+  return !(e && e[0] == '0');
+}
+
+// Adjacent loads of the current point's observations (D_LOAD of a DOBS reference, which
+// the planner places together at the start of a loop body) become D_FETCH records of up
+// to kFetchPairs asynchronous copies from the observations (flags bit 5), each record
+// committing its copies and waiting for all of them: one dispatch, the loads in flight
+// together, and no registers held for the values.  Runs on the encoded stream and
+// renumbers the loop links.
+std::vector<DInst> merge_obs_loads(const std::vector<DInst>& code) {
+  const int n = (int)code.size();
+  auto obs_load = [&](int pc) { return pc < n && code[pc].op == D_LOAD && ref_kind(code[pc].f[1]) == RK_DOBS; };
+  std::vector<DInst> out;
+  out.reserve(n);
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < n;) {
+    if (!obs_load(pc)) {
+      newpc[pc] = (int)out.size();
+      out.push_back(code[pc++]);
+      continue;
+    }
+    DInst q;
+    q.op = D_FETCH;
+    q.flags = 32 | 2 | 1;  // observation sources, commit, wait until none is pending
+    int m = 0;
+    newpc[pc] = (int)out.size();
+    while (m < kFetchPairs && obs_load(pc)) {
+      q.f[2 * m] = code[pc].f[1];
+      q.f[2 * m + 1] = code[pc].f[0];
+      newpc[pc] = (int)out.size();
+      m++;
+      pc++;
+    }
+    q.k = (uint8_t)m;
+    out.push_back(q);
+  }
+  for (DInst& d : out) {
+    if (d.op == D_LOOP) d.f[3] = newpc[d.f[3]];
+    if (d.op == D_ENDLOOP) d.f[0] = newpc[d.f[0]];
+  }
+  return out;
+}
+
 // NDVM_FMA=0 keeps the general scalar instructions instead of the fused form (a tuning knob).
 bool fma_enabled() {
   const char* e = std::getenv("NDVM_FMA");
@@ -193,6 +246,7 @@ class Planner {
   void allocate();
   void prefetch_workspace();
   void normalize_operands();
+  void hoist_seeds();
   void lower_fma();
   int const_index(double v);
   int32_t encode(const PArg& a) const;
@@ -960,11 +1014,13 @@ void Planner::normalize_operands() {
         }
         a = R(slotref(it->second));
       } else if (kind == RK_DOBS) {
+        // the point's observations load at the start of the loop body, next to each
+        // other, where merge_obs_loads packs them into fetch records
         auto it = dob.find(idx);
         if (it == dob.end()) {
           int vr = new_vr(1);
           it = dob.emplace(idx, vr).first;
-          before[pc].push_back(load(vr, src));
+          before[loop_of[pc] >= 0 ? loop_of[pc] + 1 : pc].push_back(load(vr, src));
         }
         a = R(slotref(it->second));
       } else {  // workspace value outside the prefetch
@@ -990,14 +1046,69 @@ void Planner::normalize_operands() {
   if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
 }
 
+// The reverse sweep of a data-axis body starts from the seed d(body)/d(body) = 1 at every
+// point.  When nothing in the loop writes the seed's slot (the body result feeds no
+// other body node), the seed is set once before the loop instead of once per point;
+// the allocator then keeps its slot live through the loop.  A reference other than as
+// an operand of a scalar rule, a fused update or as a reverse rule's output adjoint
+// keeps the seed in place.
+void Planner::hoist_seeds() {
+  if (!hoist_enabled()) return;
+  const int n = (int)code_.size();
+  std::vector<int> loop_of(n, -1);
+  for (int pc = 0, open = -1; pc < n; pc++) {
+    if (code_[pc].d.op == D_LOOP) { open = pc; continue; }
+    if (code_[pc].d.op == D_ENDLOOP) { open = -1; continue; }
+    loop_of[pc] = open;
+  }
+  std::vector<int> moved_to(n, -1);  // seed pc -> its loop's D_LOOP pc
+  for (int pc = 0; pc < n; pc++) {
+    const PInst& sd = code_[pc];
+    if (sd.d.op != D_SEED || loop_of[pc] < 0 || !sd.f[0].isref || sd.f[0].r.kind != RK_SLOT) continue;
+    const int vr = sd.f[0].r.id, lp = loop_of[pc];
+    auto is_vr = [&](const PArg& a) { return a.isref && a.r.kind == RK_SLOT && a.r.id == vr; };
+    bool ok = true;
+    for (const PArg& a : args_) ok = ok && !is_vr(a);
+    for (int q = lp + 1; ok && q < n && code_[q].d.op != D_ENDLOOP; q++) {
+      if (q == pc) continue;
+      const PInst& p = code_[q];
+      for (int fld = 0; ok && fld < 8; fld++) {
+        if (!is_vr(p.f[fld])) continue;
+        const bool read = slot_operand(p.d.op, fld) || (p.d.op >= B_ADD && p.d.op <= B_GRAD && fld == 0);
+        ok = read;
+      }
+    }
+    if (ok) moved_to[pc] = lp;
+  }
+  std::vector<PInst> out;
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < n; pc++) {
+    if (code_[pc].d.op == D_LOOP)
+      for (int q = pc + 1; q < n && code_[q].d.op != D_ENDLOOP; q++)
+        if (moved_to[q] == pc) out.push_back(code_[q]);
+    if (moved_to[pc] >= 0) continue;
+    newpc[pc] = (int)out.size();
+    out.push_back(code_[pc]);
+  }
+  for (PInst& p : out) {
+    if (p.d.op == D_LOOP) p.f[3] = I(newpc[p.f[3].v]);
+    if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
+  }
+  if (rev_begin_ >= 0) {
+    int r = rev_begin_;
+    while (r < n && newpc[r] < 0) r++;
+    rev_begin_ = r < n ? newpc[r] : (int)out.size();
+  }
+  code_.swap(out);
+}
+
 // Software pipeline for the reverse sweep of a spill tape.  The reverse sweep is
 // cut into windows of kFetchStride instructions; the workspace values that window k
 // reads as scalar operands are copied into a ring of slots (asynchronous copies,
 // committed as one group per window) by fetch instructions placed at the start of
-// window k - kFetchWindows, whose last one then waits until at most kFetchWindows
-// groups are pending -- so window k's values have landed when window k starts.
-// Every window commits exactly one group (possibly empty), which keeps that count
-// fixed.  The ring holds the values of any kFetchWindows + 2 consecutive windows.
+// window k - kFetchWindows; before window k starts, a wait lets only the groups
+// committed after window k's stay pending, so its values have landed.  The ring holds
+// the values of any kFetchWindows + 2 consecutive windows.
 void Planner::prefetch_workspace() {
   if (rev_begin_ < 0) return;
   const int n = (int)code_.size();
@@ -1193,6 +1304,7 @@ Plan Planner::build() {
   if (fma_enabled()) lower_fma();
   if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
   normalize_operands();
+  hoist_seeds();
   allocate();
   pl.n_slots = n_slots_;
   pl.n_save = S_;
@@ -1207,6 +1319,7 @@ Plan Planner::build() {
     pl.code.push_back(d);
   }
   for (const PArg& a : args_) pl.args.push_back(encode(a));
+  if (merge_loads_enabled()) pl.code = merge_obs_loads(pl.code);
   if (fma_enabled() && pair_enabled()) pl.code_paired = pair_fma(pl.code);
   for (const DInst& d : pl.code)
     if (d.op == D_MATMUL || d.op == D_MADD || d.op == D_MSUB || d.op == D_MSCALE || d.op == D_INV ||
@@ -1392,12 +1505,14 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
             ok = ok && ref_ok(p.args[f[1] + 3 * e], 1, true) && p.args[f[1] + 3 * e] != -1 && ref_ok(p.args[f[1] + 3 * e + 2], 1, true);
         break;
       case B_GRAD: ok = ref_ok(f[0], 1, true) && f[1] >= 0 && f[1] < p.n_params; break;
-      case D_FETCH:
-        ok = k <= kFetchPairs && ((d.flags >> 2) & 7) <= kFetchWindows;
+      case D_FETCH: {
+        const bool from_obs = d.flags & 32;
+        ok = k <= kFetchPairs && ((d.flags >> 2) & 7) <= kFetchWindows && (!from_obs || open_loop >= 0);
         for (int e = 0; ok && e < k; e++)
-          ok = ref_kind(f[2 * e]) == RK_SAVE && ref_ok(f[2 * e], 1, false) && f[2 * e + 1] != -1 &&
-               ref_ok(f[2 * e + 1], 1, true);
+          ok = ref_kind(f[2 * e]) == (from_obs ? RK_DOBS : RK_SAVE) && ref_ok(f[2 * e], 1, false) &&
+               f[2 * e + 1] != -1 && ref_ok(f[2 * e + 1], 1, true);
         break;
+      }
       default: why = "bad opcode"; return false;
     }
     const bool forward_scalar = (d.op >= D_ADD && d.op <= D_SELECT) || d.op == D_ACC;

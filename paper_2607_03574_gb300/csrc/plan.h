@@ -76,7 +76,8 @@ enum DOp : uint8_t {
   D_FETCH,          // k = count <= kFetchPairs; pairs (f0 workspace ref, f1 slot), (f2, f3), ...:
                     // asynchronous copies into slots; flags bit1: then commit the copies issued
                     // since the last commit as one group; bit0: then wait until at most n groups
-                    // are pending, n = flags bits 2..4 (<= kFetchWindows)
+                    // are pending, n = flags bits 2..4 (<= kFetchWindows); bit5: the sources are
+                    // observations of the current data point (DOBS refs, inside a data-axis loop)
   // ---- fused multiply-add form of the cheap scalar rules ----
   D_FMA,            // slot f0 = (is_zero(slot f4) ? slot f3 : fma(+-slot f1, slot f2, slot f3)), f5 save;
                     // flags bit0 negates the first factor.  f4 is the zero-skip test (an adjoint

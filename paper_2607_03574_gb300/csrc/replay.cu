@@ -410,11 +410,12 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       // asynchronous copies of workspace values into slots (the owner of element 0
       // copies; the warp barrier after the wait publishes them to the group)
       // (unrolled: the record's fields stay in registers only when indexed by constants)
+      // (flags bit 5: the sources are observations of the current data point)
       if (L.own(0))
 #pragma unroll
         for (int e = 0; e < kFetchPairs; e++) {
           if (e >= in.k) break;
-          const T* src = L.savep(f[2 * e]);
+          const T* src = (in.flags & 32) ? L.obs + L.dbase + (f[2 * e] & kRefIndexMask) : L.savep(f[2 * e]);
           const unsigned dst = (unsigned)__cvta_generic_to_shared(L.wp(f[2 * e + 1]));
           if (sizeof(T) == 8)
             asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(src) : "memory");
