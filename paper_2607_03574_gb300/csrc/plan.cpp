@@ -105,6 +105,12 @@ bool hoist_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_COALESCE=0 keeps every adjoint copy as its own instruction (a tuning knob).
+bool coalesce_enabled() {
+  const char* e = std::getenv("NDVM_COALESCE");
+  return !(e && e[0] == '0');
+}
+
 // NDVM_MERGELOADS=0 keeps one record per observation load (a tuning knob).
 bool merge_loads_enabled() {
   const char* e = std::getenv("NDVM_MERGELOADS");
@@ -247,6 +253,7 @@ class Planner {
   void prefetch_workspace();
   void normalize_operands();
   void hoist_seeds();
+  void coalesce_copies();
   void lower_fma();
   int const_index(double v);
   int32_t encode(const PArg& a) const;
@@ -1046,6 +1053,93 @@ void Planner::normalize_operands() {
   if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
 }
 
+// A first adjoint contribution that is a plain copy (a sum's rule passes its output
+// adjoint g on unchanged: slot d = g * 1 + (-0)) needs no instruction when d can share
+// g's slot: g is written no more after the copy, every later read of g comes no later
+// than the first later write of d, and both live in the same place (the same data-axis
+// loop body, or outside every loop, so that no loop repeats a read after a write).  The
+// copy is then dropped and d renamed to g.  A zero g is the one value whose bits can
+// differ: the copy gives -0, the shared slot keeps g's sign of zero.  Scalar slots only;
+// one referenced from an argument list stays.
+void Planner::coalesce_copies() {
+  if (!coalesce_enabled()) return;
+  const int n = (int)code_.size();
+  const int mzero = const_index(-0.0);
+  std::vector<int> loop_of(n, -1);
+  for (int pc = 0, open = -1; pc < n; pc++) {
+    if (code_[pc].d.op == D_LOOP) { open = pc; continue; }
+    if (code_[pc].d.op == D_ENDLOOP) { open = -1; continue; }
+    loop_of[pc] = open;
+  }
+  struct Use { int pc; bool read; };
+  const int nv = (int)vrs_.size();
+  std::vector<std::vector<Use>> uses(nv);
+  std::vector<char> in_args(nv, 0), scalar(nv, 0);
+  for (int v = 0; v < nv; v++) scalar[v] = vrs_[v].width == 1;
+  auto vr_of = [](const PArg& a) { return (a.isref && a.r.kind == RK_SLOT) ? a.r.id : -1; };
+  for (const PArg& a : args_) if (vr_of(a) >= 0) in_args[vr_of(a)] = 1;
+  for (int pc = 0; pc < n; pc++) {
+    const PInst& p = code_[pc];
+    for (int fld = 0; fld < 8; fld++) {
+      const int v = vr_of(p.f[fld]);
+      if (v < 0) continue;
+      if (p.f[fld].r.off != 0) scalar[v] = 0;
+      const bool read = slot_operand(p.d.op, fld) || (p.d.op >= B_ADD && p.d.op <= B_GRAD && fld == 0);
+      uses[v].push_back({pc, read});
+    }
+  }
+  std::vector<int> rename(nv, -1);
+  auto root = [&](int v) {
+    if (v < 0) return v;
+    while (rename[v] >= 0) v = rename[v];
+    return v;
+  };
+  std::vector<char> drop(n, 0);
+  auto is_const = [](const PArg& a, int idx) { return a.isref && a.r.kind == RK_CONST && a.r.id + a.r.off == idx; };
+  for (int pc = 0; pc < n; pc++) {
+    const PInst& c = code_[pc];
+    if (c.d.op != D_FMA || c.d.flags != 0 || !is_const(c.f[2], one_const_) || !is_const(c.f[3], mzero)) continue;
+    if (c.f[5].isref || (c.f[5].v != -1)) continue;
+    const int d = root(vr_of(c.f[0])), g = root(vr_of(c.f[1]));
+    if (d < 0 || g < 0 || d == g || root(vr_of(c.f[4])) != g || !scalar[d] || !scalar[g] || in_args[d] || in_args[g])
+      continue;
+    const int here = loop_of[pc];
+    bool ok = true;
+    int first_write_d = INT_MAX;
+    for (const Use& u : uses[d]) {
+      if (u.pc == pc) continue;
+      ok = ok && u.pc > pc && loop_of[u.pc] == here;
+      if (!u.read) first_write_d = std::min(first_write_d, u.pc);
+    }
+    for (const Use& u : uses[g]) {
+      if (u.pc == pc) continue;
+      ok = ok && loop_of[u.pc] == here;
+      if (u.pc > pc) ok = ok && u.read && u.pc <= first_write_d;
+    }
+    if (!ok) continue;
+    drop[pc] = 1;
+    rename[d] = g;
+    for (const Use& u : uses[d]) if (u.pc != pc) uses[g].push_back(u);
+    uses[d].clear();
+  }
+  std::vector<PInst> out;
+  std::vector<int> newpc(n, -1);
+  for (int pc = 0; pc < n; pc++) {
+    newpc[pc] = (int)out.size();
+    if (drop[pc]) continue;
+    PInst p = code_[pc];
+    for (int fld = 0; fld < 8; fld++)
+      if (vr_of(p.f[fld]) >= 0) p.f[fld].r.id = root(p.f[fld].r.id);
+    out.push_back(p);
+  }
+  for (PInst& p : out) {
+    if (p.d.op == D_LOOP) p.f[3] = I(newpc[p.f[3].v]);
+    if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
+  }
+  if (rev_begin_ >= 0 && rev_begin_ < n) rev_begin_ = newpc[rev_begin_];
+  code_.swap(out);
+}
+
 // The reverse sweep of a data-axis body starts from the seed d(body)/d(body) = 1 at every
 // point.  When nothing in the loop writes the seed's slot (the body result feeds no
 // other body node), the seed is set once before the loop instead of once per point;
@@ -1303,6 +1397,7 @@ Plan Planner::build() {
   }
   if (fma_enabled()) lower_fma();
   if (grad_ && spill_ && prefetch_enabled()) prefetch_workspace();
+  if (fma_enabled()) coalesce_copies();
   normalize_operands();
   hoist_seeds();
   allocate();

@@ -403,19 +403,23 @@ def test_shared_point_values_match_per_lane_values(ndvm, oracle_mod, cuda, monke
 
 @pytest.mark.parametrize("cfg,B", [(3, 16384), (4, 8192), (6, 256)])
 def test_paired_chains_and_trimmed_fetches_are_exact(ndvm, oracle_mod, cuda, monkeypatch, cfg, B):
-    """Two stream rewrites change no arithmetic: pairing a fused update with the next one
+    """Three stream rewrites change no arithmetic: sharing a slot between an adjoint and
+    its first contribution when that is a plain copy (equal values; only a zero's sign
+    may differ, and zeros compare equal), pairing a fused update with the next one
     that reads its result (two contributions to one adjoint, a step of a recurrence), and
     leaving out the fetch records of reverse-sweep windows that fetch nothing (waits then
-    count only the groups that were committed). The replay with both equals, bit for bit,
-    the replay without them (independent pairs only, a commit and a wait in every window),
+    count only the groups that were committed). The replay with them equals the replay
+    without them (copies kept, independent pairs only, a commit and a wait in every window),
     at the launch shape the bench uses, and the oracle at 1e-12 on sampled lanes."""
     import torch
     w = W.config(cfg, B=B)
     monkeypatch.setenv("NDVM_DEPPAIR", "0")
     monkeypatch.setenv("NDVM_FETCHTRIM", "0")
+    monkeypatch.setenv("NDVM_COALESCE", "0")
     plain = ndvm.trace_build(w.program, w.frontend)
     monkeypatch.delenv("NDVM_DEPPAIR")
     monkeypatch.delenv("NDVM_FETCHTRIM")
+    monkeypatch.delenv("NDVM_COALESCE")
     tape = ndvm.trace_build(w.program, w.frontend)
     p = torch.tensor(w.params, device="cuda")
     o = torch.tensor(w.obs, device="cuda")
@@ -441,18 +445,21 @@ def _region_workloads():
 
 @pytest.mark.parametrize("k", range(8))
 def test_point_loads_and_hoisted_seed_are_exact(ndvm, oracle_mod, cuda, monkeypatch, k):
-    """Two rewrites of data-axis loops change no arithmetic: the current point's
-    observations load at the start of the loop body as asynchronous copies, up to four
-    per record, and the reverse sweep's seed d(body)/d(body) = 1 is set once before the
-    loop when nothing in the body writes its slot. The replay with both equals, bit for
-    bit, the replay without them, and the oracle at 1e-12 on sampled lanes."""
+    """Rewrites of data-axis loops change no arithmetic: the current point's observations
+    load at the start of the loop body as asynchronous copies, up to four per record; the
+    reverse sweep's seed d(body)/d(body) = 1 is set once before the loop when nothing in
+    the body writes its slot; an adjoint whose first contribution is a plain copy shares
+    the copied slot. The replay with them equals the replay without them (a zero's sign
+    may differ; zeros compare equal), and the oracle at 1e-12 on sampled lanes."""
     import torch
     w = _region_workloads()[k]
     monkeypatch.setenv("NDVM_MERGELOADS", "0")
     monkeypatch.setenv("NDVM_HOIST", "0")
+    monkeypatch.setenv("NDVM_COALESCE", "0")
     plain = ndvm.trace_build(w.program, w.frontend)
     monkeypatch.delenv("NDVM_MERGELOADS")
     monkeypatch.delenv("NDVM_HOIST")
+    monkeypatch.delenv("NDVM_COALESCE")
     tape = ndvm.trace_build(w.program, w.frontend)
     p = torch.tensor(w.params, device="cuda")
     o = torch.tensor(w.obs, device="cuda")
