@@ -979,9 +979,9 @@ void Planner::lower_fma() {
 // Load-store form: every operand that slot_operand() marks is made a slot.  A
 // constant, parameter or observation is loaded once into a slot before its first
 // use -- before the enclosing data-axis loop when the use is inside one -- and the
-// slot stays live to its last use; a per-point observation is loaded inside the loop
-// body before its first use there; a workspace value not covered by the prefetch is
-// loaded right before its use.
+// slot stays live to its last use; a per-point observation is loaded at the start of
+// the loop body; a workspace value not covered by the prefetch is loaded right before
+// its use.
 void Planner::normalize_operands() {
   const int n = (int)code_.size();
   std::vector<int> loop_of(n, -1);  // enclosing D_LOOP pc
@@ -1053,14 +1053,27 @@ void Planner::normalize_operands() {
   if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
 }
 
-// A first adjoint contribution that is a plain copy (a sum's rule passes its output
-// adjoint g on unchanged: slot d = g * 1 + (-0)) needs no instruction when d can share
-// g's slot: g is written no more after the copy, every later read of g comes no later
-// than the first later write of d, and both live in the same place (the same data-axis
-// loop body, or outside every loop, so that no loop repeats a read after a write).  The
-// copy is then dropped and d renamed to g.  A zero g is the one value whose bits can
-// differ: the copy gives -0, the shared slot keeps g's sign of zero.  Scalar slots only;
-// one referenced from an argument list stays.
+// A first adjoint contribution that is a plain copy needs no work when the new adjoint
+// d can share the slots of the copied adjoint g: a sum's scalar rule (d = g * 1 + (-0)),
+// and the first target of a matrix sum's or difference's rule (d = gZ; also the second
+// target of a sum).  Conditions: g is written no more after the copy, every later read
+// of g comes no later than the first later write of d, d is not referenced before the
+// copy, both have the same width, neither appears in an argument list, and both live
+// in the same place (the same data-axis loop body, or outside every loop, so that no
+// loop repeats a read after a write).  The copy is then dropped (a matrix rule keeps
+// its other target) and d renamed to g.  A zero is the one value whose bits can
+// differ: the copy gives -0 (or +0), the shared slot keeps g's sign of zero.
+namespace {
+// whether field `fld` of an instruction with opcode `op` only reads its slot reference
+// (a conservative answer: false for every field that may be written)
+bool reads_only(int op, int fld) {
+  if (op >= B_ADD && op <= B_GRAD) return fld == 0 || fld >= 3;  // gz and primal inputs; f1, f2 targets
+  if (op == D_FETCH || fld == 0) return false;                    // destinations
+  if ((op == D_SIN || op == D_COS || op == D_DET || op == D_LOGDET) && fld == 4) return false;  // aux outputs
+  return true;
+}
+}  // namespace
+
 void Planner::coalesce_copies() {
   if (!coalesce_enabled()) return;
   const int n = (int)code_.size();
@@ -1071,21 +1084,17 @@ void Planner::coalesce_copies() {
     if (code_[pc].d.op == D_ENDLOOP) { open = -1; continue; }
     loop_of[pc] = open;
   }
-  struct Use { int pc; bool read; };
+  struct Use { int pc, fld; bool read; };
   const int nv = (int)vrs_.size();
   std::vector<std::vector<Use>> uses(nv);
-  std::vector<char> in_args(nv, 0), scalar(nv, 0);
-  for (int v = 0; v < nv; v++) scalar[v] = vrs_[v].width == 1;
+  std::vector<char> in_args(nv, 0);
   auto vr_of = [](const PArg& a) { return (a.isref && a.r.kind == RK_SLOT) ? a.r.id : -1; };
   for (const PArg& a : args_) if (vr_of(a) >= 0) in_args[vr_of(a)] = 1;
   for (int pc = 0; pc < n; pc++) {
     const PInst& p = code_[pc];
     for (int fld = 0; fld < 8; fld++) {
       const int v = vr_of(p.f[fld]);
-      if (v < 0) continue;
-      if (p.f[fld].r.off != 0) scalar[v] = 0;
-      const bool read = slot_operand(p.d.op, fld) || (p.d.op >= B_ADD && p.d.op <= B_GRAD && fld == 0);
-      uses[v].push_back({pc, read});
+      if (v >= 0) uses[v].push_back({pc, fld, reads_only(p.d.op, fld)});
     }
   }
   std::vector<int> rename(nv, -1);
@@ -1094,33 +1103,53 @@ void Planner::coalesce_copies() {
     while (rename[v] >= 0) v = rename[v];
     return v;
   };
-  std::vector<char> drop(n, 0);
-  auto is_const = [](const PArg& a, int idx) { return a.isref && a.r.kind == RK_CONST && a.r.id + a.r.off == idx; };
-  for (int pc = 0; pc < n; pc++) {
+  // try to let the adjoint in field tf of instruction pc share the slots of the one in
+  // field sf (the instruction's other references to g: the fields in also_g)
+  auto try_merge = [&](int pc, int tf, int sf, int also_g) -> bool {
     const PInst& c = code_[pc];
-    if (c.d.op != D_FMA || c.d.flags != 0 || !is_const(c.f[2], one_const_) || !is_const(c.f[3], mzero)) continue;
-    if (c.f[5].isref || (c.f[5].v != -1)) continue;
-    const int d = root(vr_of(c.f[0])), g = root(vr_of(c.f[1]));
-    if (d < 0 || g < 0 || d == g || root(vr_of(c.f[4])) != g || !scalar[d] || !scalar[g] || in_args[d] || in_args[g])
-      continue;
+    const int d = root(vr_of(c.f[tf])), g = root(vr_of(c.f[sf]));
+    if (d < 0 || g < 0 || d == g || vrs_[d].width != vrs_[g].width || in_args[d] || in_args[g]) return false;
+    if (c.f[tf].r.off != 0 || c.f[sf].r.off != 0) return false;
     const int here = loop_of[pc];
-    bool ok = true;
     int first_write_d = INT_MAX;
     for (const Use& u : uses[d]) {
-      if (u.pc == pc) continue;
-      ok = ok && u.pc > pc && loop_of[u.pc] == here;
+      if (u.pc == pc && u.fld == tf) continue;
+      if (u.pc <= pc || loop_of[u.pc] != here) return false;
       if (!u.read) first_write_d = std::min(first_write_d, u.pc);
     }
     for (const Use& u : uses[g]) {
-      if (u.pc == pc) continue;
-      ok = ok && loop_of[u.pc] == here;
-      if (u.pc > pc) ok = ok && u.read && u.pc <= first_write_d;
+      if (u.pc == pc) {
+        if (u.fld == sf || u.fld == also_g) continue;
+        return false;
+      }
+      if (loop_of[u.pc] != here) return false;
+      if (u.pc > pc && (!u.read || u.pc > first_write_d)) return false;
     }
-    if (!ok) continue;
-    drop[pc] = 1;
     rename[d] = g;
-    for (const Use& u : uses[d]) if (u.pc != pc) uses[g].push_back(u);
+    for (const Use& u : uses[d])
+      if (!(u.pc == pc && u.fld == tf)) uses[g].push_back(u);
     uses[d].clear();
+    return true;
+  };
+  auto is_const = [](const PArg& a, int idx) { return a.isref && a.r.kind == RK_CONST && a.r.id + a.r.off == idx; };
+  std::vector<char> drop(n, 0);
+  for (int pc = 0; pc < n; pc++) {
+    PInst& c = code_[pc];
+    if (c.d.op == D_FMA) {
+      if (c.d.flags != 0 || !is_const(c.f[2], one_const_) || !is_const(c.f[3], mzero)) continue;
+      if (c.f[5].isref || c.f[5].v != -1 || root(vr_of(c.f[4])) != root(vr_of(c.f[1]))) continue;
+      if (try_merge(pc, 0, 1, 4)) drop[pc] = 1;
+    } else if (c.d.op == B_MADD || c.d.op == B_MSUB) {
+      if ((c.d.flags & 1) && try_merge(pc, 1, 0, -1)) {
+        c.f[1] = I(-1);
+        c.d.flags &= (uint8_t)~1u;
+      }
+      if (c.d.op == B_MADD && (c.d.flags & 2) && try_merge(pc, 2, 0, -1)) {
+        c.f[2] = I(-1);
+        c.d.flags &= (uint8_t)~2u;
+      }
+      if (vr_of(c.f[1]) < 0 && vr_of(c.f[2]) < 0) drop[pc] = 1;
+    }
   }
   std::vector<PInst> out;
   std::vector<int> newpc(n, -1);
