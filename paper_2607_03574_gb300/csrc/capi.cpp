@@ -2,6 +2,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -132,7 +133,24 @@ constexpr size_t kSmemLimit = 227 * 1024;
 // bounds: 128 per thread for the element-split and staged variants, 64 otherwise)
 constexpr size_t kSmemPerSm = 228 * 1024, kSmemPerBlockReserved = 1024;
 constexpr int kRegsPerSm = 65536, kMaxRegsStagedOrShared = 128, kMaxRegsPlain = 64;
-constexpr int64_t kNumSms = 152;
+// SMs of the current device, which the launch heuristics size grids by (152 on GB300,
+// also the answer when no device responds); cached per device
+int64_t num_sms() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return 152;
+  }
+  int n = cache[dev].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return 152;
+  }
+  cache[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
 // threads of a block that serves a single lane (block-cooperative matrix tapes)
 constexpr int kBlockLaneThreads = 256;
 // lanes per launch when a workspace is used: the kernel indexes a lane's workspace
@@ -178,13 +196,14 @@ int ilog2(int g) {
 
 Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
   Shape s;
+  const int64_t sms = num_sms();
   const int ov = threads_per_lane_override();
   if (p.has_regions && p.n_save == 0) {
     // data-axis tapes: a lane's points split over a thread group, one slot column per thread
     int g = ov;
     if (!g) {
       g = 1;
-      while (g < 32 && B * g < kNumSms * 256) g *= 2;
+      while (g < 32 && B * g < sms * 256) g *= 2;
     }
     s.log2g = ilog2(g);
     while (s.tpb > 32 && (size_t)p.n_slots * s.tpb * elem > kSmemLimit) s.tpb /= 2;
@@ -196,7 +215,7 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     int g = ov > 16 ? 16 : ov;
     if (!g) {
       int gf = 1, gs = 1;
-      while (gf < 16 && B * gf < kNumSms * 4 * 64) gf *= 2;
+      while (gf < 16 && B * gf < sms * 4 * 64) gf *= 2;
       while (gs < 16 && (size_t)p.n_slots * (128 / gs + 1) * elem > kSmemLimit / 4) gs *= 2;
       g = gf > gs ? gf : gs;
     }
@@ -228,7 +247,7 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
   // blocks an SM would hold at most: the grid's blocks spread over the SMs
   const int64_t lanes_per_block = s.tpb >> s.log2g;
   const int64_t grid = (B + lanes_per_block - 1) / lanes_per_block;
-  const int want = (int)std::min<int64_t>((grid + kNumSms - 1) / kNumSms, 64);
+  const int want = (int)std::min<int64_t>((grid + sms - 1) / sms, 64);
   auto resident = [&](size_t bytes, bool staged) { return std::min(blocks_per_sm(bytes, staged), want); };
   const size_t staged_smem = (s.smem + 15) / 16 * 16 + stage_bytes;
   if (stage_enabled() && !p.has_regions && p.code.size() > 2 * (size_t)kStageChunk && staged_smem <= kSmemLimit &&
