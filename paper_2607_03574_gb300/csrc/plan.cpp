@@ -52,13 +52,21 @@ bool pair_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_SAVEPAIR=0 leaves fused instructions that save their result unpaired (a tuning
+// knob).
+bool save_pair_enabled() {
+  const char* e = std::getenv("NDVM_SAVEPAIR");
+  return !(e && e[0] == '0');
+}
+
 // NDVM_DEPPAIR=0 pairs independent fused instructions only (a tuning knob).
 bool dep_pair_enabled() {
   const char* e = std::getenv("NDVM_DEPPAIR");
   return !(e && e[0] == '0');
 }
 
-// Two adjacent D_FMA records without saves become one D_FMA2: one dispatch for both.
+// Two adjacent D_FMA records become one D_FMA2: one dispatch for both (a save's
+// workspace index travels in 24 bits of the record).
 // Runs on the encoded stream (physical slots).  The kernel loads every operand of the
 // pair before it stores either result, so a second destination that the first reads
 // is safe.  When the second reads the first's result (a chain, e.g. two contributions
@@ -68,19 +76,28 @@ bool dep_pair_enabled() {
 std::vector<DInst> pair_fma(const std::vector<DInst>& code) {
   const int n = (int)code.size();
   const bool dep_ok = dep_pair_enabled();
+  const bool save_pairs = save_pair_enabled();
   std::vector<DInst> out;
   out.reserve(n);
   std::vector<int> newpc(n, -1);
   for (int pc = 0; pc < n; pc++) {
     const DInst& a = code[pc];
     newpc[pc] = (int)out.size();
-    if (pc + 1 < n && a.op == D_FMA && code[pc + 1].op == D_FMA && a.f[5] == -1 && code[pc + 1].f[5] == -1) {
+    auto save24 = [&](int32_t sv) { return sv == -1 || (sv >= 0 && sv < kNoSave24 && save_pairs); };
+    if (pc + 1 < n && a.op == D_FMA && code[pc + 1].op == D_FMA && save24(a.f[5]) && save24(code[pc + 1].f[5])) {
       const DInst& b = code[pc + 1];
       const bool raw = b.f[1] == a.f[0] || b.f[2] == a.f[0] || b.f[3] == a.f[0] || b.f[4] == a.f[0];
       if (raw ? dep_ok : b.f[0] != a.f[0]) {
         DInst q;
         q.op = D_FMA2;
-        q.flags = (uint8_t)((a.flags & 1) | ((b.flags & 1) << 1) | (raw ? 4 : 0));
+        const bool saves = a.f[5] != -1 || b.f[5] != -1;
+        q.flags = (uint8_t)((a.flags & 1) | ((b.flags & 1) << 1) | (raw ? 4 : 0) | (saves ? 8 : 0));
+        if (saves) {
+          const uint32_t s1 = a.f[5] == -1 ? (uint32_t)kNoSave24 : (uint32_t)a.f[5];
+          const uint32_t s2 = b.f[5] == -1 ? (uint32_t)kNoSave24 : (uint32_t)b.f[5];
+          q.r = (uint8_t)s1; q.c = (uint8_t)(s1 >> 8); q.k = (uint8_t)(s1 >> 16);
+          q.pad0 = (uint8_t)s2; q.pad1 = (uint8_t)(s2 >> 8); q.pad2 = (uint8_t)(s2 >> 16);
+        }
         for (int k = 0; k < 5; k++) q.f[k] = a.f[k];
         q.f[5] = b.f[0]; q.f[6] = b.f[1]; q.f[7] = b.f[2]; q.pad3 = b.f[3]; q.pad4 = b.f[4];
         out.push_back(q);
@@ -1526,8 +1543,9 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
     const int32_t* f = d.f;
     const int r = d.r, c = d.c, k = d.k, w = r * c, n = d.r;
     bool ok = true;
-    if (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim || ((d.op == D_MATMUL || d.op == B_MATMUL) && (k < 1 || k > kMaxDim)) ||
-        (d.op == D_CMP && k > 4)) {
+    // (a paired update's r, c and k bytes hold a save index, not a shape)
+    if ((d.op != D_FMA2 && (r < 1 || c < 1 || r > kMaxDim || c > kMaxDim)) ||
+        ((d.op == D_MATMUL || d.op == B_MATMUL) && (k < 1 || k > kMaxDim)) || (d.op == D_CMP && k > 4)) {
       why = "bad shape";
       return false;
     }
@@ -1581,6 +1599,10 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
       case D_LOAD: ok = ref_ok(f[0], 1, true) && f[1] != -1 && ref_ok(f[1], 1, false); break;
       case D_FMA2:
         ok = f[0] != -1 && f[5] != -1 && ref_ok(f[0], 1, true) && ref_ok(f[5], 1, true);
+        if (d.flags & 8) {
+          const int32_t s1 = d.r | (d.c << 8) | (d.k << 16), s2 = d.pad0 | (d.pad1 << 8) | (d.pad2 << 16);
+          ok = ok && (s1 == kNoSave24 || save_ok(s1, 1)) && (s2 == kNoSave24 || save_ok(s2, 1));
+        }
         for (int q = 1; q <= 4; q++) ok = ok && f[q] != -1 && ref_ok(f[q], 1, true);
         ok = ok && f[6] != -1 && f[7] != -1 && d.pad3 != -1 && d.pad4 != -1 && ref_ok(f[6], 1, true) &&
              ref_ok(f[7], 1, true) && ref_ok(d.pad3, 1, true) && ref_ok(d.pad4, 1, true);

@@ -86,7 +86,9 @@ enum DOp : uint8_t {
   D_FMA2,           // two D_FMA without saves in one record: (f0 dst, f1, f2, f3, f4 zero-skip)
                     // and (f5 dst, f6, f7, pad3, pad4 zero-skip); flags bit0 / bit1 negate the first
                     // factor of the first / second; bit2: the second's operands that name f0 read
-                    // the first's result
+                    // the first's result; bit3: saves, the first's workspace index in bytes
+                    // (r, c, k) and the second's in (pad0, pad1, pad2), 24 bits little-endian,
+                    // kNoSave24 for none
   D_NOPS
 };
 
@@ -101,6 +103,9 @@ bool slot_operand(int op, int field);
 constexpr int kFetchPairs = 4;
 constexpr int kFetchStride = 4;
 constexpr int kFetchWindows = 4;
+
+// "no save" in the 24-bit save fields of D_FMA2
+constexpr int32_t kNoSave24 = 0xFFFFFF;
 
 // 48 bytes, 16-byte aligned (three 128-bit words; staged copies move 16-byte pieces).
 struct alignas(16) DInst {

@@ -403,6 +403,11 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
       const T z2 = is_zero(g2) ? c2 : fma(x2, y2, c2);
       L.st(f[0], 0, z1);
       L.st(f[5], 0, z2);
+      if (in.flags & 8) {  // saves: 24-bit workspace indices in (r, c, k) and (pad0, pad1, pad2)
+        const int32_t s1 = in.r | (in.c << 8) | (in.k << 16), s2 = in.pad0 | (in.pad1 << 8) | (in.pad2 << 16);
+        if (s1 != kNoSave24) L.save_out(s1, 0, z1);
+        if (s2 != kNoSave24) L.save_out(s2, 0, z2);
+      }
       if (sync_each) group_sync();
       continue;
     }

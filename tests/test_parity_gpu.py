@@ -405,19 +405,23 @@ def test_shared_point_values_match_per_lane_values(ndvm, oracle_mod, cuda, monke
 def test_paired_chains_and_trimmed_fetches_are_exact(ndvm, oracle_mod, cuda, monkeypatch, cfg, B):
     """Three stream rewrites change no arithmetic: sharing a slot between an adjoint and
     its first contribution when that is a plain copy (equal values; only a zero's sign
-    may differ, and zeros compare equal), pairing a fused update with the next one
+    may differ, and zeros compare equal), pairing fused updates that save their result,
+    pairing a fused update with the next one
     that reads its result (two contributions to one adjoint, a step of a recurrence), and
     leaving out the fetch records of reverse-sweep windows that fetch nothing (waits then
     count only the groups that were committed). The replay with them equals the replay
-    without them (copies kept, independent pairs only, a commit and a wait in every window),
+    without them (copies kept, independent pairs without saves only, a commit and a wait in
+    every window),
     at the launch shape the bench uses, and the oracle at 1e-12 on sampled lanes."""
     import torch
     w = W.config(cfg, B=B)
     monkeypatch.setenv("NDVM_DEPPAIR", "0")
+    monkeypatch.setenv("NDVM_SAVEPAIR", "0")
     monkeypatch.setenv("NDVM_FETCHTRIM", "0")
     monkeypatch.setenv("NDVM_COALESCE", "0")
     plain = ndvm.trace_build(w.program, w.frontend)
     monkeypatch.delenv("NDVM_DEPPAIR")
+    monkeypatch.delenv("NDVM_SAVEPAIR")
     monkeypatch.delenv("NDVM_FETCHTRIM")
     monkeypatch.delenv("NDVM_COALESCE")
     tape = ndvm.trace_build(w.program, w.frontend)
