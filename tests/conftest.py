@@ -89,3 +89,26 @@ def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol, mag=None):
             bad.append("non-finite gradient class mismatch")
     return (not bad), {"worst_loss": worst_l, "worst_grad": worst_g, "nonfinite_lanes": int((~fin).sum()),
                        "problems": bad}
+
+
+# hand-derived fixtures under tests/golden (each cites the rule it exercises and shows
+# its derivation)
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+def golden_cases():
+    return sorted(f for f in os.listdir(GOLDEN) if f.endswith(".json"))
+
+
+def load_golden(name):
+    import json
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def golden_close(got, want, tol):
+    """Exact equality when tol == 0, else |got - want| <= tol * |want| element by element."""
+    got, want = np.asarray(got, dtype=np.float64), np.asarray(want, dtype=np.float64)
+    if tol == 0:
+        return np.array_equal(got, want)
+    return bool(np.all(np.abs(got - want) <= tol * np.maximum(np.abs(want), 1e-300)))

@@ -8,10 +8,12 @@ other on every workload.
 """
 import math
 
+
 import numpy as np
 import pytest
 
 import workloads as W
+from conftest import golden_cases, golden_close, load_golden
 
 REV, DUAL, VAL = 0 + 1, 2, 0
 
@@ -483,3 +485,19 @@ def test_second_client_workloads(oracle_mod):
     text = W.bytecode_w3(2).replace("PARAM 1\nADD\nTANH", "PUSH 0.5\nADD\nTANH")
     _, g = run(oracle_mod, text, np.array([[0.3, 2.0], [1.0, 50.0]]), np.array([0.1, 0.2]), frontend=1)
     np.testing.assert_array_equal(g[:, 1], 0.0)
+
+
+@pytest.mark.parametrize("name", golden_cases())
+def test_golden_fixtures(oracle_mod, name):
+    """Hand-derived values (each fixture cites the adjoint rule it exercises and shows the
+    derivation): the oracle's reverse mode and its dual numbers both reproduce them,
+    exactly where every intermediate is exact in binary64, else within the fixture's
+    tolerance (a correctly rounded logarithm)."""
+    g = load_golden(name)
+    fe = oracle_mod.FRONTEND_BYTECODE if g["frontend"] == "bytecode" else oracle_mod.FRONTEND_SCHEME
+    params = np.array(g["params"], dtype=np.float64)
+    obs = np.array(g["obs"], dtype=np.float64)
+    for mode in (oracle_mod.MODE_REVERSE, oracle_mod.MODE_DUAL):
+        loss, grad = oracle_mod.run(g["program"], params, obs, frontend=fe, mode=mode)
+        assert golden_close(loss, g["loss"], g["tol"]), (name, mode, loss)
+        assert golden_close(grad, g["grad"], g["tol"]), (name, mode, grad)
