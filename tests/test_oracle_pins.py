@@ -501,3 +501,21 @@ def test_golden_fixtures(oracle_mod, name):
         loss, grad = oracle_mod.run(g["program"], params, obs, frontend=fe, mode=mode)
         assert golden_close(loss, g["loss"], g["tol"]), (name, mode, loss)
         assert golden_close(grad, g["grad"], g["tol"]), (name, mode, grad)
+
+
+def test_integer_helpers_and_stack_ops(oracle_mod):
+    """The oracle's surface for the structural helpers and the bytecode stack moves, at
+    values fixed by arithmetic: 7 quotient 2 + 7 remainder 3 + the third of (4 5 6) = 10,
+    so L = 10 a; expt a 3 = a^3 with derivative 3 a^2; (p1 - p0)^2 after SWAP, SUB."""
+    p = np.array([[2.0], [-0.5]])
+    loss, grad = oracle_mod.run("(model (params a) (* a (exact->inexact (+ (quotient 7 2) (remainder 7 3) "
+                                "(list-ref (list 4 5 6) 2)))))", p, np.zeros(0))
+    np.testing.assert_array_equal(loss, [20.0, -5.0])
+    np.testing.assert_array_equal(grad, [[10.0], [10.0]])
+    loss, grad = oracle_mod.run("(model (params a) (expt a 3))", p, np.zeros(0))
+    np.testing.assert_array_equal(loss, [8.0, -0.125])
+    np.testing.assert_array_equal(grad, [[12.0], [0.75]])
+    loss, grad = oracle_mod.run("PARAM 0\nPARAM 1\nSWAP\nSUB\nPOWI 2\n", np.array([[1.0, 4.0]]), np.zeros(0),
+                                frontend=oracle_mod.FRONTEND_BYTECODE)
+    np.testing.assert_array_equal(loss, [9.0])
+    np.testing.assert_array_equal(grad, [[-6.0, 6.0]])

@@ -205,3 +205,16 @@ def test_structural_surface_records_only_numeric_primitives(ndvm):
     lst = ("(define (sum l) (if (null? l) 0.0 (+ (car l) (sum (cdr l))))) "
            "(model (params a b) (sum (list a b (* a b))))")
     assert ndvm.trace_build(lst).info()["n_nodes"] == 3 + 1 + 3       # 0.0, a, b; a*b; three sums
+
+
+def test_integer_helpers_and_stack_ops_record_only_numbers(ndvm):
+    """quotient, remainder, list-ref and exact->inexact are structural (one constant node
+    for the number they produce); expt with an integer exponent is the integer power;
+    the bytecode's SWAP moves stack entries and POWI n records one node."""
+    t = ndvm.trace_build("(model (params a) (* a (exact->inexact (+ (quotient 7 2) (remainder 7 3) "
+                         "(list-ref (list 4 5 6) 2)))))")
+    assert t.serialize() == encode(1, 0, 2, [N("param"), N("const"), N("mul", 0, 1)], [10.0])
+    t = ndvm.trace_build("(model (params a) (expt a 3))")
+    assert t.serialize() == encode(1, 0, 1, [N("param"), N("powi", 0, imm=3)])
+    t = ndvm.trace_build("PARAM 0\nPARAM 1\nSWAP\nSUB\nPOWI 2\n", ndvm.FE_BYTECODE)
+    assert t.serialize() == encode(2, 0, 3, [N("param"), N("param", imm=1), N("sub", 1, 0), N("powi", 2, imm=2)])
