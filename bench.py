@@ -175,7 +175,8 @@ def cpu_sample_lanes(args, progs):
     return 2048 if args.config == 2 else progs[0].B
 
 
-def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = False, min_seconds: float = 0.0):
+def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = False, min_seconds: float = 0.0,
+                       tile: bool = True):
     """Time the oracle on a bounded sample: `lanes_per_prog` lanes of every program,
     repeated until at least `min_seconds` have passed (small workloads)."""
     import oracle
@@ -185,7 +186,7 @@ def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = Fa
     while True:
         for w in progs:
             p = w.params[:lanes_per_prog]
-            if len(p) < 1024:  # small populations: tile the lanes so thread start-up does not dominate
+            if tile and len(p) < 1024:  # small populations: tile the lanes so thread start-up does not dominate
                 p = np.resize(p, (1024, p.shape[1]))
             if f32:
                 p = p.astype(np.float32).astype(np.float64)
@@ -193,6 +194,26 @@ def oracle_sample_time(progs, lanes_per_prog: int, nthreads: int, f32: bool = Fa
             n += len(p)
         if time.perf_counter() - t0 >= min_seconds:
             return n, time.perf_counter() - t0
+
+
+def cpu_baseline(args, progs):
+    """The oracle timed on the host cores: every core on a bounded sample (about 10-30 s
+    of CPU work), and one core on a sample sized from that rate to take about 2 s."""
+    cores = os.cpu_count() or 1
+    f32 = args.dtype == "f32"
+    lanes = cpu_sample_lanes(args, progs)
+    oracle_sample_time(progs[:2], 2, cores, f32)
+    n, dt = oracle_sample_time(progs, lanes, cores, f32, min_seconds=2.0)
+    rate = n / dt
+    per_core = rate / cores
+    progs1 = progs[:max(1, min(len(progs), 8))]
+    lanes1 = int(min(lanes, max(1, per_core * 2.0 / len(progs1))))
+    n1, dt1 = oracle_sample_time(progs1, lanes1, 1, f32, min_seconds=0.5, tile=False)
+    return {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{lanes} lanes of each of the {len(progs)} program(s), repeated to {n} lane evals ({dt:.1f} s)",
+            "single_core": {"value": n1 / dt1, "unit": UNIT, "cores": 1,
+                            "sample": f"{lanes1} lanes of each of {len(progs1)} program(s), repeated to {n1} lane "
+                                      f"evals ({dt1:.1f} s)"}}
 
 
 def run_reference(args):
@@ -395,14 +416,7 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        cores = os.cpu_count() or 1
-        f32 = args.dtype == "f32"
-        lanes = cpu_sample_lanes(args, progs)
-        oracle_sample_time(progs[:2], 2, cores, f32)
-        n, dt = oracle_sample_time(progs, lanes, cores, f32, min_seconds=2.0)
-        cpu = {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{lanes} lanes of each of the {len(progs)} program(s), repeated to {n} lane evals "
-                         f"({dt:.1f} s)"}
+        cpu = cpu_baseline(args, progs)
 
     if rank == 0:
         line = {

@@ -44,3 +44,19 @@ def test_warmup_below_three_is_refused():
     r = run_bench(["--impl", "reference", "--config", "1", "--steps", "1", "--warmup", "1"])
     assert r.returncode != 0
     assert "warmup" in r.stderr
+
+
+def test_cpu_baseline_times_all_cores_and_one():
+    """The GPU arm's cpu_baseline: the oracle on every host core, and on one core over a
+    sample sized from the all-core rate (a bounded run)."""
+    import importlib.util
+    import types
+    spec = importlib.util.spec_from_file_location("bench_mod", os.path.join(ROOT, "bench.py"))
+    b = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(b)
+    args = types.SimpleNamespace(config=1, lanes=0, programs=1, dtype="f64", cpu_lanes=0)
+    progs, _ = b.workload_for(args, b.SEED)
+    cb = b.cpu_baseline(args, progs)
+    assert cb["kind"] == "oracle" and cb["unit"] == b.UNIT and cb["cores"] >= 1 and cb["value"] > 0
+    one = cb["single_core"]
+    assert one["cores"] == 1 and one["value"] > 0 and one["unit"] == b.UNIT and one["sample"]
