@@ -28,7 +28,7 @@
  *     derivatives (dual numbers, the method section 6 uses for its hand-compiled
  *     Kalman ceiling).
  *
- * Readings of points the paper leaves open (all listed in the design doc):
+ * Readings of points the paper leaves open (the GPU path takes the same ones):
  *   R1  tanh, neg, select, compare, param/obs loads and matrix add/sub/scale are
  *       not in Appendix C: tanh' = 1 - z^2, neg' = -1, select passes the adjoint
  *       to the branch the lane took (section 6: only lanes that took a side send
@@ -713,7 +713,7 @@ static double* gbuf_sel(Ctx* cx, Num* n, int absmode) {
 /* absmode = 1 runs the same propagation on absolute values (|g| times |local
  * derivative|, every contribution added): the result bounds the magnitude of the
  * terms summed into each gradient component, the scale against which rounding
- * in any summation order is judged. */
+ * in any summation order is measured. */
 static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
   /* post-order over dependent nodes */
   size_t cap = 1024, cnt = 0, sp = 0;

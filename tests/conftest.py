@@ -52,7 +52,7 @@ def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol, mag=None):
     s_k = max(max_j |ora gradient_j| of that lane, mag_k), where mag_k (from the oracle's
     magnitude mode) is the component propagated through absolute values -- the size of
     the terms it sums.  A component that is a small difference of large terms is thus
-    judged against those terms, the scale any summation order's rounding is bounded by.  A lane whose oracle loss is non-finite must be non-finite
+    measured against those terms, the scale any summation order's rounding is bounded by.  A lane whose oracle loss is non-finite must be non-finite
     in the same class (NaN vs +-inf) on the GPU and is excluded from the relative checks.
     Returns (ok, report).
     """
