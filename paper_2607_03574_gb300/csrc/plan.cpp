@@ -1120,6 +1120,13 @@ void Planner::coalesce_copies() {
     while (rename[v] >= 0) v = rename[v];
     return v;
   };
+  // whether an instruction may read g and write d when the two share slots: it must
+  // read every element it needs before it stores any (the fused form loads all its
+  // operands first; the scalar rules read their adjoint once; the matrix sum's rule
+  // reads and writes the same element), which a product's or a scatter's rule does not
+  auto reads_before_writes = [](int op) {
+    return op == D_FMA || op == B_MADD || op == B_MSUB || (op >= B_ADD && op <= B_POWI) || op == B_SELECT;
+  };
   // try to let the adjoint in field tf of instruction pc share the slots of the one in
   // field sf (the instruction's other references to g: the fields in also_g)
   auto try_merge = [&](int pc, int tf, int sf, int also_g) -> bool {
@@ -1134,6 +1141,11 @@ void Planner::coalesce_copies() {
       if (u.pc <= pc || loop_of[u.pc] != here) return false;
       if (!u.read) first_write_d = std::min(first_write_d, u.pc);
     }
+    // the instruction that first writes d after the copy may also read g (the slot
+    // then holds g's value, which is d's); only one that reads before it writes may
+    if (first_write_d != INT_MAX && !reads_before_writes(code_[first_write_d].d.op))
+      for (int fld = 0; fld < 8; fld++)
+        if (root(vr_of(code_[first_write_d].f[fld])) == g) return false;
     for (const Use& u : uses[g]) {
       if (u.pc == pc) {
         if (u.fld == sf || u.fld == also_g) continue;

@@ -112,3 +112,22 @@ def golden_close(got, want, tol):
     if tol == 0:
         return np.array_equal(got, want)
     return bool(np.all(np.abs(got - want) <= tol * np.maximum(np.abs(want), 1e-300)))
+
+
+# Programs where an input's adjoint and the output adjoint it copies could share slots
+# while a product's or a transpose's rule reads the one and writes the other: the
+# slots must stay apart there (the rule reads elements it has already written).
+HAZARDS = {
+    "transpose_sum": "(model (params a b c) (let* ((B (matrix 2 2 a b c a)) (A (transpose B)) (Z (m+ A B))) "
+                     "(trace (matmul Z Z))))",
+    "matmul_sum": "(model (params a b c) (let* ((B (matrix 2 2 a b c a)) (C (matrix 2 2 1.5 0.5 -0.25 2.0)) "
+                  "(A (matmul B C)) (Z (m+ A B))) (trace (matmul Z Z))))",
+    "scalar_sum": "(model (params a b c) (let* ((x (* a b)) (z (+ x a c))) (* z z)))",
+}
+
+
+def hazard_workloads():
+    import workloads as _W
+    rng = np.random.default_rng(5)
+    return [_W.Workload(name, text, 0, rng.normal(size=(8, 3)), np.zeros(0), np.zeros(3))
+            for name, text in HAZARDS.items()]

@@ -4,16 +4,21 @@
 // instruction semantics (plan.h): slot files, the fused multiply-add form and its
 // paired record, data-axis loops, shared per-point values, workspace saves and
 // fetches (a fetch copies at once; the device's later wait then has nothing to wait
-// for), first-contribution stores and exact-zero adjoint skips.  Matrix instructions
-// are not simulated (exit status 3).
+// for), first-contribution stores and exact-zero adjoint skips, and the matrix
+// instructions (element e of a matrix operand is element ref + e; products accumulate
+// left to right with fused multiply-adds; inverses and determinants by closed forms to
+// 3 x 3, Gauss-Jordan elimination with partial pivoting above).  An instruction the
+// executor does not know ends the run with exit status 3.
 //
 // Input on stdin:  frontend B P n_obs stream(0 plain, 1 paired) / B*P params / n_obs obs /
 //                  the program text up to end of input.
 // Output: one line per lane: the loss and the P gradient components as C hex floats.
+// (The executor takes G = 1: one thread owns every element of its lane.)
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
 #include <iostream>
+#include <utility>
 #include <sstream>
 #include <string>
 #include <vector>
@@ -32,6 +37,58 @@ double powi_rep(double a, int n) {
   double z = a;
   for (int i = 1; i < n; i++) z = z * a;
   return z;
+}
+
+// determinant and (optionally) inverse of the n x n matrix a (row-major)
+double det_inv(const std::vector<double>& a, int n, std::vector<double>* inv) {
+  if (n == 1) {
+    if (inv) (*inv)[0] = 1.0 / a[0];
+    return a[0];
+  }
+  if (n == 2) {
+    const double d = a[0] * a[3] - a[1] * a[2];
+    if (inv) {
+      const double r = 1.0 / d;
+      (*inv)[0] = a[3] * r; (*inv)[1] = -a[1] * r; (*inv)[2] = -a[2] * r; (*inv)[3] = a[0] * r;
+    }
+    return d;
+  }
+  if (n == 3) {
+    const double c00 = a[4] * a[8] - a[5] * a[7], c01 = a[5] * a[6] - a[3] * a[8], c02 = a[3] * a[7] - a[4] * a[6];
+    const double d = a[0] * c00 + a[1] * c01 + a[2] * c02;
+    if (inv) {
+      const double c10 = a[2] * a[7] - a[1] * a[8], c11 = a[0] * a[8] - a[2] * a[6], c12 = a[1] * a[6] - a[0] * a[7];
+      const double c20 = a[1] * a[5] - a[2] * a[4], c21 = a[2] * a[3] - a[0] * a[5], c22 = a[0] * a[4] - a[1] * a[3];
+      const double r = 1.0 / d;
+      const double cof[9] = {c00, c10, c20, c01, c11, c21, c02, c12, c22};
+      for (int e = 0; e < 9; e++) (*inv)[e] = cof[e] * r;
+    }
+    return d;
+  }
+  std::vector<std::vector<double>> w(n, std::vector<double>(2 * n));
+  for (int i = 0; i < n; i++)
+    for (int j = 0; j < 2 * n; j++) w[i][j] = j < n ? a[i * n + j] : (j - n == i ? 1.0 : 0.0);
+  double d = 1.0;
+  for (int col = 0; col < n; col++) {
+    int piv = col;
+    for (int i = col + 1; i < n; i++)
+      if (std::fabs(w[i][col]) > std::fabs(w[piv][col])) piv = i;
+    if (piv != col) { std::swap(w[piv], w[col]); d = -d; }
+    const double pv = w[col][col];
+    d = d * pv;
+    const double r = 1.0 / pv;
+    for (int j = 0; j < 2 * n; j++) w[col][j] = w[col][j] * r;
+    for (int i = 0; i < n; i++) {
+      if (i == col) continue;
+      const double fct = w[i][col];
+      if (fct != 0.0)
+        for (int j = 0; j < 2 * n; j++) w[i][j] = w[i][j] - fct * w[col][j];
+    }
+  }
+  if (inv)
+    for (int i = 0; i < n; i++)
+      for (int j = 0; j < n; j++) (*inv)[i * n + j] = w[i][n + j];
+  return d;
 }
 
 struct Unsupported {};
@@ -68,6 +125,43 @@ struct Run {
   }
   void save_out(int32_t sidx, double v) {
     if (sidx >= 0) save[(int64_t)sidx * save_ld + col] = v;
+  }
+  // element e of a (matrix) operand, and of a slot range
+  double el(int32_t ref, int e) {
+    const int32_t i = ref_index(ref) + e;
+    switch (ref_kind(ref)) {
+      case RK_SLOT: return s[(size_t)i];
+      case RK_CONST: return consts[(size_t)i];
+      case RK_OBS: return obs[i];
+      case RK_DOBS: return obs[dbase + i];
+      case RK_SAVE: return save[(int64_t)i * save_ld + col];
+      default: return params[i];
+    }
+  }
+  double& sel(int32_t ref, int e) { return s[(size_t)(ref_index(ref) + e)]; }
+  void upd_el(int32_t ref, int e, double v, bool first) {
+    double& q = sel(ref, e);
+    q = first ? v : q + v;
+  }
+  void zero_first(int32_t ref, int w, bool first) {
+    if (first && ref != -1)
+      for (int e = 0; e < w; e++) sel(ref, e) = 0.0;
+  }
+  bool all_zero(int32_t gz, int w) {
+    for (int e = 0; e < w; e++)
+      if (!is_zero(sel(gz, e))) return false;
+    return true;
+  }
+  // a[0] b[0] + a[sa] b[sb] + ... over n terms, left to right, fused after the first
+  double dot(int32_t ra, int ea, int sa, int32_t rb, int eb, int sb, int n) {
+    double acc = el(ra, ea) * el(rb, eb);
+    for (int q = 1; q < n; q++) acc = std::fma(el(ra, ea + q * sa), el(rb, eb + q * sb), acc);
+    return acc;
+  }
+  std::vector<double> mat(int32_t ref, int w) {
+    std::vector<double> m((size_t)w);
+    for (int e = 0; e < w; e++) m[(size_t)e] = el(ref, e);
+    return m;
   }
   void upd(int32_t ref, double v, bool first) {
     double& q = slot(ref);
@@ -167,6 +261,167 @@ struct Run {
           const double z = !is_zero(ld(f[1])) ? ld(f[2]) : ld(f[4]);
           slot(f[0]) = z;
           save_out(f[3], z);
+          break;
+        }
+        case D_GATHER: {
+          const int32_t* g = p.args.data() + f[1];
+          for (int e = 0; e < f[2]; e++) {
+            const double v = ld(g[e]);
+            sel(f[0], e) = v;
+            save_out(f[3] < 0 ? -1 : f[3] + e, v);
+          }
+          break;
+        }
+        case D_MADD: case D_MSUB: case D_MSCALE: {
+          const int w = in.r * in.c;
+          const double sc = in.op == D_MSCALE ? ld(f[1]) : 0.0;
+          for (int e = 0; e < w; e++) {
+            const double z = in.op == D_MADD ? el(f[1], e) + el(f[2], e)
+                             : in.op == D_MSUB ? el(f[1], e) - el(f[2], e) : sc * el(f[2], e);
+            sel(f[0], e) = z;
+            save_out(f[3] < 0 ? -1 : f[3] + e, z);
+          }
+          break;
+        }
+        case D_MATMUL: {
+          const int r = in.r, c = in.c, kk = in.k;
+          std::vector<double> z((size_t)(r * c));
+          for (int i = 0; i < r; i++)
+            for (int j = 0; j < c; j++) z[(size_t)(i * c + j)] = dot(f[1], i * kk, 1, f[2], j, c, kk);
+          for (int e = 0; e < r * c; e++) {
+            sel(f[0], e) = z[(size_t)e];
+            save_out(f[3] < 0 ? -1 : f[3] + e, z[(size_t)e]);
+          }
+          break;
+        }
+        case D_INV: {
+          const int n = in.r;
+          std::vector<double> inv((size_t)(n * n));
+          det_inv(mat(f[1], n * n), n, &inv);
+          for (int e = 0; e < n * n; e++) {
+            sel(f[0], e) = inv[(size_t)e];
+            save_out(f[3] < 0 ? -1 : f[3] + e, inv[(size_t)e]);
+          }
+          break;
+        }
+        case D_DET: case D_LOGDET: {
+          const int n = in.r;
+          const bool aux = f[4] != -1 || f[5] >= 0;
+          std::vector<double> inv((size_t)(n * n));
+          const double dt = det_inv(mat(f[1], n * n), n, aux ? &inv : nullptr);
+          const double z = in.op == D_DET ? dt : std::log(dt);
+          slot(f[0]) = z;
+          save_out(f[3], z);
+          if (aux)
+            for (int e = 0; e < n * n; e++) {
+              if (f[4] != -1) sel(f[4], e) = inv[(size_t)e];
+              save_out(f[5] < 0 ? -1 : f[5] + e, inv[(size_t)e]);
+            }
+          break;
+        }
+        case D_TRACE: {
+          const int n = in.r;
+          double t = el(f[1], 0);
+          for (int i = 1; i < n; i++) t = t + el(f[1], i * n + i);
+          slot(f[0]) = t;
+          break;
+        }
+        case B_GATHER: {
+          const int32_t* g = p.args.data() + f[1];
+          const bool z = all_zero(f[0], f[2]);
+          for (int e = 0; e < f[2]; e++) {
+            const int32_t t = g[2 * e];
+            if (t == -1) continue;
+            const bool first = g[2 * e + 1] != 0;
+            if (z) zero_if_first(t, first);
+            else upd(t, sel(f[0], e), first);
+          }
+          break;
+        }
+        case B_SCATTER: {
+          if (f[1] == -1) break;
+          zero_first(f[1], f[4], in.flags & 1);
+          if (all_zero(f[0], f[2])) break;
+          const int32_t* m = p.args.data() + f[3];
+          for (int e = 0; e < f[2]; e++) sel(f[1], m[e]) = sel(f[1], m[e]) + sel(f[0], e);
+          break;
+        }
+        case B_MADD: case B_MSUB: {
+          const int w = in.r * in.c;
+          const bool fa = in.flags & 1, fb = in.flags & 2;
+          if (all_zero(f[0], w)) { zero_first(f[1], w, fa); zero_first(f[2], w, fb); break; }
+          for (int e = 0; e < w; e++) {
+            const double g = sel(f[0], e);
+            if (f[1] != -1) upd_el(f[1], e, g, fa);
+            if (f[2] != -1) upd_el(f[2], e, in.op == B_MADD ? g : -g, fb);
+          }
+          break;
+        }
+        case B_MSCALE: {
+          const int w = in.r * in.c;
+          const bool fa = in.flags & 1, fb = in.flags & 2;
+          if (all_zero(f[0], w)) { zero_first(f[1], 1, fa); zero_first(f[2], w, fb); break; }
+          if (f[1] != -1) {
+            double acc = sel(f[0], 0) * el(f[4], 0);
+            for (int e = 1; e < w; e++) acc = std::fma(sel(f[0], e), el(f[4], e), acc);
+            upd(f[1], acc, fa);
+          }
+          if (f[2] != -1) {
+            const double sc = ld(f[3]);
+            for (int e = 0; e < w; e++) upd_el(f[2], e, sc * sel(f[0], e), fb);
+          }
+          break;
+        }
+        case B_MATMUL: {
+          const int r = in.r, c = in.c, kk = in.k;
+          const bool fa = in.flags & 1, fb = in.flags & 2;
+          if (all_zero(f[0], r * c)) { zero_first(f[1], r * kk, fa); zero_first(f[2], kk * c, fb); break; }
+          // element by element, each update stored before the next element is computed
+          // (the device's order)
+          if (f[1] != -1)  // gA (r x k) += gZ (r x c) B^T
+            for (int i = 0; i < r; i++)
+              for (int q = 0; q < kk; q++) upd_el(f[1], i * kk + q, dot(f[0], i * c, 1, f[4], q * c, 1, c), fa);
+          if (f[2] != -1)  // gB (k x c) += A^T gZ
+            for (int q = 0; q < kk; q++)
+              for (int j = 0; j < c; j++) upd_el(f[2], q * c + j, dot(f[3], q, kk, f[0], j, c, r), fb);
+          break;
+        }
+        case B_INV: {
+          const int n = in.r;
+          const bool fa = in.flags & 1;
+          if (f[1] == -1) break;
+          if (all_zero(f[0], n * n)) { zero_first(f[1], n * n, fa); break; }
+          std::vector<double> m((size_t)(n * n));  // M = gZ B^T, B the saved inverse
+          for (int pp = 0; pp < n; pp++)
+            for (int j = 0; j < n; j++) m[(size_t)(pp * n + j)] = dot(f[0], pp * n, 1, f[5], j * n, 1, n);
+          for (int e = 0; e < n * n; e++) {  // gA -= B^T M
+            const int i = e / n, j = e - i * n;
+            double acc = el(f[5], i) * m[(size_t)j];
+            for (int pp = 1; pp < n; pp++) acc = std::fma(el(f[5], pp * n + i), m[(size_t)(pp * n + j)], acc);
+            upd_el(f[1], e, -acc, fa);
+          }
+          break;
+        }
+        case B_DET: case B_LOGDET: {
+          const int n = in.r;
+          const bool fa = in.flags & 1;
+          if (f[1] == -1) break;
+          const double g = slot(f[0]);
+          if (is_zero(g)) { zero_first(f[1], n * n, fa); break; }
+          const double fac = in.op == B_DET ? g * ld(f[5]) : g;
+          for (int e = 0; e < n * n; e++) {
+            const int i = e / n, j = e - i * n;
+            upd_el(f[1], e, fac * el(f[6], j * n + i), fa);
+          }
+          break;
+        }
+        case B_TRACE: {
+          const int n = in.r;
+          if (f[1] == -1) break;
+          const double g = slot(f[0]);
+          zero_first(f[1], n * n, in.flags & 1);
+          if (is_zero(g)) break;
+          for (int i = 0; i < n; i++) sel(f[1], i * n + i) = sel(f[1], i * n + i) + g;
           break;
         }
         case D_ZERO:

@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import golden_cases, golden_close, load_golden, rel_check
+from conftest import golden_cases, golden_close, hazard_workloads, load_golden, rel_check
 
 pytestmark = pytest.mark.gpu
 
@@ -502,3 +502,26 @@ def test_golden_fixtures_gpu(ndvm, cuda, name):
     assert golden_close(loss.cpu().numpy(), g["loss"], tol), (name, loss)
     assert golden_close(fl.cpu().numpy(), g["loss"], tol), (name, fl)
     assert golden_close(grad.cpu().numpy(), g["grad"], tol), (name, grad)
+
+
+def test_shared_adjoint_slots_stay_apart_where_a_rule_reads_after_writing(ndvm, oracle_mod, cuda, monkeypatch):
+    """Z = A + B with A = B^T (or A = B C): the sum's rule copies Z's adjoint to both A and
+    B, and the transpose's (product's) rule then reads A's adjoint while it writes B's.
+    Sharing one slot there would let the rule read elements it has already written, so
+    the planner keeps those adjoints apart: the replay equals the one without slot
+    sharing and the oracle."""
+    import torch
+    for w in hazard_workloads():
+        tape = ndvm.trace_build(w.program)
+        monkeypatch.setenv("NDVM_COALESCE", "0")
+        plain = ndvm.trace_build(w.program)
+        monkeypatch.delenv("NDVM_COALESCE")
+        p = torch.tensor(w.params, device="cuda")
+        o = torch.zeros(1, dtype=torch.float64, device="cuda")
+        l1, g1 = ndvm.value_and_grad(tape, p, o)
+        l2, g2 = ndvm.value_and_grad(plain, p, o)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(l1.cpu().numpy(), l2.cpu().numpy())
+        np.testing.assert_array_equal(g1.cpu().numpy(), g2.cpu().numpy())
+        ol, og, om = oracle_run(oracle_mod, w)
+        check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og, om)

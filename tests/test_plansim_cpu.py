@@ -17,7 +17,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import rel_check
+from conftest import hazard_workloads, rel_check
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 CSRC = os.path.join(ROOT, "paper_2607_03574_gb300", "csrc")
@@ -54,7 +54,7 @@ def simulate(exe, w, stream=0, env_extra=None):
 
 
 def programs():
-    ws = [W.config(1)]
+    ws = hazard_workloads() + [W.config(1)]
     ws += W.random_exprs(6, B=48, n_points=32, seed=99)
     ws += W.control_fuzz(24, B=24)
     ws += W.second_client(B=24)
