@@ -1,8 +1,7 @@
 """The planner's stream rewrites checked without a GPU.
 
 tests/plansim.cpp executes the replay plans on the CPU with the device interpreter's
-instruction semantics (scalar and data-axis tapes; matrix instructions are not
-simulated). For every program: the simulated replay matches the oracle under the
+instruction semantics (scalar, data-axis and matrix tapes, one thread per lane). For every program: the simulated replay matches the oracle under the
 parity rule, the paired stream gives the same values as the unpaired one, and the
 plans built with every rewrite switched off give the same values as the default plans
 (copies coalesced, seeds hoisted, observation loads merged, dependent and saving pairs,
@@ -59,6 +58,9 @@ def programs():
     ws += W.control_fuzz(24, B=24)
     ws += W.second_client(B=24)
     ws.append(W.logistic(B=12))
+    ws.append(W.kalman_cv4(B=6, T=12))
+    ws.append(W.kalman_rand8(B=4, T=6))
+    ws.append(W.kalman_highd(B=2, D=12, m=3, T=3))
     return ws
 
 
@@ -78,3 +80,56 @@ def test_simulated_plans_match_the_oracle_and_each_other(plansim, oracle_mod, k)
         other = simulate(plansim, w, stream, env)
         assert np.array_equal(other[0], base[0]), (w.name, stream, env)
         assert np.array_equal(other[1], base[1]), (w.name, stream, env)
+
+
+def matrix_program(rng, n_params=4):
+    """A seeded program over small matrices: let*-bound intermediates that later terms
+    reuse (sums of a matrix and its own transposes, products, scalings), reduced by
+    trace, element reference, determinant and log-determinant of well-conditioned
+    matrices. Text only."""
+    n = int(rng.integers(2, 4))
+    p = [f"p{i}" for i in range(n_params)]
+
+    def leaf():
+        return "(matrix {n} {n} {els})".format(n=n, els=" ".join(
+            str(rng.choice(p)) if rng.random() < 0.6 else repr(round(float(rng.normal()), 3)) for _ in range(n * n)))
+
+    binds, names = [], []
+    for i in range(int(rng.integers(3, 6))):
+        pool = names or [leaf()]
+        a = str(rng.choice(pool)) if names else leaf()
+        b = str(rng.choice(names)) if names and rng.random() < 0.7 else leaf()
+        kind = rng.integers(0, 8)
+        expr = {0: f"(m+ {a} {b})", 1: f"(m- {a} {b})", 2: f"(matmul {a} {b})", 3: f"(transpose {a})",
+                4: f"(mscale {rng.choice(p)} {a})", 5: f"(m+ {a} (transpose {a}))",
+                6: f"(m+ (transpose {a}) {a})", 7: f"(m+ (matmul {a} {b}) {a})"}[int(kind)]
+        names.append(f"M{i}")
+        binds.append(f"(M{i} {expr})")
+    terms = []
+    for m in names[-3:]:
+        spd = f"(m+ (matmul {m} (transpose {m})) (identity {n}))"
+        terms += [f"(trace {m})", f"(mref {m} 0 {n - 1})", f"(logdet {spd})", f"(trace (inv {spd}))",
+                  f"(* 0.1 (det {m}))"]
+    body = " ".join(str(t) for t in rng.choice(terms, size=4, replace=False))
+    return f"(model (params {' '.join(p)}) (let* ({' '.join(binds)}) (+ {body})))"
+
+
+MATRIX_CASES = [matrix_program(np.random.default_rng(1000 + i)) for i in range(60)]
+
+
+@pytest.mark.parametrize("k", range(len(MATRIX_CASES)))
+def test_simulated_matrix_programs(plansim, oracle_mod, k):
+    """Seeded matrix programs (the adjoint slots of sums, transposes and products meet
+    in many ways): the simulated replay matches the oracle, with and without the
+    rewrites, on the plain and the paired stream. (A determinant of a singular matrix
+    gives a NaN gradient through A^-T on both sides; NaNs compare equal here.)"""
+    rng = np.random.default_rng(k)
+    w = W.Workload(f"matrix_{k}", MATRIX_CASES[k], 0, rng.normal(0.0, 0.5, (6, 4)), np.zeros(0), np.zeros(4))
+    base = simulate(plansim, w, 0)
+    ol, og, om = oracle_mod.run(w.program, w.params, w.obs, magnitudes=True)
+    ok, rep = rel_check(base[0], base[1], ol, og, 1e-12, om)
+    assert ok, (w.program, rep)
+    for stream, env in ((1, None), (0, OFF), (1, OFF)):
+        other = simulate(plansim, w, stream, env)
+        assert np.array_equal(other[0], base[0], equal_nan=True), (w.program, stream, env)
+        assert np.array_equal(other[1], base[1], equal_nan=True), (w.program, stream, env)
