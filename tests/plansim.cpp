@@ -10,7 +10,8 @@
 // 3 x 3, Gauss-Jordan elimination with partial pivoting above).  An instruction the
 // executor does not know ends the run with exit status 3.
 //
-// Input on stdin:  frontend B P n_obs stream(0 plain, 1 paired) / B*P params / n_obs obs /
+// Input on stdin:  frontend B P n_obs stream(0 plain, 1 paired, 2 the value-only plan) / B*P params /
+//                  n_obs obs /
 //                  the program text up to end of input.
 // Output: one line per lane: the loss and the P gradient components as C hex floats.
 // (The executor takes G = 1: one thread owns every element of its lane.)
@@ -533,7 +534,7 @@ int main() {
     if (fe == 0) trace_scheme(text.data(), text.size(), b, err);
     else trace_bytecode(text.data(), text.size(), b, err);
     if (b.t.loss < 0) { std::fprintf(stderr, "no result: %s\n", err.c_str()); return 2; }
-    const Plan p = make_plan(b.t, true);
+    const Plan p = make_plan(b.t, stream != 2);  // stream 2: the value-only plan
     std::string why;
     if (!validate_plan(p, b.t.consts.size(), why)) { std::fprintf(stderr, "plan check: %s\n", why.c_str()); return 4; }
     std::vector<double> consts = b.t.consts;

@@ -76,6 +76,8 @@ def test_simulated_plans_match_the_oracle_and_each_other(plansim, oracle_mod, k)
     ol, og, om = oracle_mod.run(w.program, w.params, w.obs, frontend=w.frontend, magnitudes=True)
     ok, rep = rel_check(base[0], base[1], ol, og, 1e-12, om)
     assert ok, (w.name, rep)
+    value = simulate(plansim, w, 2)
+    assert np.array_equal(value[0], base[0]), w.name  # the value-only plan gives the same loss bits
     for stream, env in ((1, None), (0, OFF), (1, OFF)):
         other = simulate(plansim, w, stream, env)
         assert np.array_equal(other[0], base[0]), (w.name, stream, env)
