@@ -131,3 +131,35 @@ def hazard_workloads():
     rng = np.random.default_rng(5)
     return [_W.Workload(name, text, 0, rng.normal(size=(8, 3)), np.zeros(0), np.zeros(3))
             for name, text in HAZARDS.items()]
+
+
+def matrix_program(rng, n_params=4):
+    """A seeded program over small matrices: let*-bound intermediates that later terms
+    reuse (sums of a matrix and its own transposes, products, scalings), reduced by
+    trace, element reference, determinant and log-determinant of well-conditioned
+    matrices. Text only."""
+    n = int(rng.integers(2, 4))
+    p = [f"p{i}" for i in range(n_params)]
+
+    def leaf():
+        return "(matrix {n} {n} {els})".format(n=n, els=" ".join(
+            str(rng.choice(p)) if rng.random() < 0.6 else repr(round(float(rng.normal()), 3)) for _ in range(n * n)))
+
+    binds, names = [], []
+    for i in range(int(rng.integers(3, 6))):
+        pool = names or [leaf()]
+        a = str(rng.choice(pool)) if names else leaf()
+        b = str(rng.choice(names)) if names and rng.random() < 0.7 else leaf()
+        kind = rng.integers(0, 8)
+        expr = {0: f"(m+ {a} {b})", 1: f"(m- {a} {b})", 2: f"(matmul {a} {b})", 3: f"(transpose {a})",
+                4: f"(mscale {rng.choice(p)} {a})", 5: f"(m+ {a} (transpose {a}))",
+                6: f"(m+ (transpose {a}) {a})", 7: f"(m+ (matmul {a} {b}) {a})"}[int(kind)]
+        names.append(f"M{i}")
+        binds.append(f"(M{i} {expr})")
+    terms = []
+    for m in names[-3:]:
+        spd = f"(m+ (matmul {m} (transpose {m})) (identity {n}))"
+        terms += [f"(trace {m})", f"(mref {m} 0 {n - 1})", f"(logdet {spd})", f"(trace (inv {spd}))",
+                  f"(* 0.1 (det {m}))"]
+    body = " ".join(str(t) for t in rng.choice(terms, size=4, replace=False))
+    return f"(model (params {' '.join(p)}) (let* ({' '.join(binds)}) (+ {body})))"

@@ -519,3 +519,18 @@ def test_integer_helpers_and_stack_ops(oracle_mod):
                                 frontend=oracle_mod.FRONTEND_BYTECODE)
     np.testing.assert_array_equal(loss, [9.0])
     np.testing.assert_array_equal(grad, [[-6.0, 6.0]])
+
+
+def test_matrix_programs_reverse_equals_dual_numbers(oracle_mod):
+    """Seeded programs over small matrices (sums, differences, products, transposes,
+    scalings, inverses, determinants, log-determinants, traces, element references,
+    with reused intermediates): the oracle's reverse mode agrees with its dual numbers
+    (two independent derivative engines) under the parity rule."""
+    from conftest import matrix_program, rel_check
+    for i in range(40):
+        prog = matrix_program(np.random.default_rng(7000 + i))
+        params = np.random.default_rng(i).normal(0.0, 0.5, (4, 4))
+        lr, gr, mr = oracle_mod.run(prog, params, np.zeros(0), magnitudes=True)
+        ld, gd = oracle_mod.run(prog, params, np.zeros(0), mode=oracle_mod.MODE_DUAL)
+        ok, rep = rel_check(lr, gr, ld, gd, 1e-12, mr)
+        assert ok, (prog, rep)

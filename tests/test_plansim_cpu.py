@@ -16,7 +16,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import hazard_workloads, rel_check
+from conftest import hazard_workloads, matrix_program, rel_check
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 CSRC = os.path.join(ROOT, "paper_2607_03574_gb300", "csrc")
@@ -82,38 +82,6 @@ def test_simulated_plans_match_the_oracle_and_each_other(plansim, oracle_mod, k)
         other = simulate(plansim, w, stream, env)
         assert np.array_equal(other[0], base[0]), (w.name, stream, env)
         assert np.array_equal(other[1], base[1]), (w.name, stream, env)
-
-
-def matrix_program(rng, n_params=4):
-    """A seeded program over small matrices: let*-bound intermediates that later terms
-    reuse (sums of a matrix and its own transposes, products, scalings), reduced by
-    trace, element reference, determinant and log-determinant of well-conditioned
-    matrices. Text only."""
-    n = int(rng.integers(2, 4))
-    p = [f"p{i}" for i in range(n_params)]
-
-    def leaf():
-        return "(matrix {n} {n} {els})".format(n=n, els=" ".join(
-            str(rng.choice(p)) if rng.random() < 0.6 else repr(round(float(rng.normal()), 3)) for _ in range(n * n)))
-
-    binds, names = [], []
-    for i in range(int(rng.integers(3, 6))):
-        pool = names or [leaf()]
-        a = str(rng.choice(pool)) if names else leaf()
-        b = str(rng.choice(names)) if names and rng.random() < 0.7 else leaf()
-        kind = rng.integers(0, 8)
-        expr = {0: f"(m+ {a} {b})", 1: f"(m- {a} {b})", 2: f"(matmul {a} {b})", 3: f"(transpose {a})",
-                4: f"(mscale {rng.choice(p)} {a})", 5: f"(m+ {a} (transpose {a}))",
-                6: f"(m+ (transpose {a}) {a})", 7: f"(m+ (matmul {a} {b}) {a})"}[int(kind)]
-        names.append(f"M{i}")
-        binds.append(f"(M{i} {expr})")
-    terms = []
-    for m in names[-3:]:
-        spd = f"(m+ (matmul {m} (transpose {m})) (identity {n}))"
-        terms += [f"(trace {m})", f"(mref {m} 0 {n - 1})", f"(logdet {spd})", f"(trace (inv {spd}))",
-                  f"(* 0.1 (det {m}))"]
-    body = " ".join(str(t) for t in rng.choice(terms, size=4, replace=False))
-    return f"(model (params {' '.join(p)}) (let* ({' '.join(binds)}) (+ {body})))"
 
 
 MATRIX_CASES = [matrix_program(np.random.default_rng(1000 + i)) for i in range(60)]
