@@ -1074,10 +1074,11 @@ void Planner::normalize_operands() {
 // d can share the slots of the copied adjoint g: a sum's scalar rule (d = g * 1 + (-0)),
 // and the first target of a matrix sum's or difference's rule (d = gZ; also the second
 // target of a sum).  Conditions: g is written no more after the copy, every later read
-// of g comes no later than the first later write of d, d is not referenced before the
-// copy, both have the same width, neither appears in an argument list, and both live
-// in the same place (the same data-axis loop body, or outside every loop, so that no
-// loop repeats a read after a write).  The copy is then dropped (a matrix rule keeps
+// of g comes no later than the first later write of d, that first writer reads every
+// element it needs before it stores any if it also reads g, d is not referenced before
+// the copy, both have the same width, neither appears in an argument list, and both
+// live in the same place (the same data-axis loop body, or outside every loop, so that
+// no loop repeats a read after a write).  The copy is then dropped (a matrix rule keeps
 // its other target) and d renamed to g.  A zero is the one value whose bits can
 // differ: the copy gives -0 (or +0), the shared slot keeps g's sign of zero.
 namespace {
