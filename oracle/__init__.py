@@ -53,7 +53,7 @@ def _load():
             f.restype = ctypes.c_int
             f.argtypes = [ctypes.c_char_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_longlong, ctypes.c_int,
                           ctypes.c_void_p, ctypes.c_longlong, ctypes.c_void_p, ctypes.c_void_p,
-                          ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_char_p,
+                          ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_char_p,
                           ctypes.c_size_t]
             _lib = lib
     return _lib
@@ -64,12 +64,10 @@ class OracleError(RuntimeError):
 
 
 def run(program: str, params, obs, *, frontend: int = FRONTEND_SCHEME, mode: int = MODE_REVERSE,
-        nthreads: int = 1, magnitudes: bool = False, f32: bool = False):
+        nthreads: int = 1, f32: bool = False):
     """Evaluate every lane.  params: (B, P) float64; obs: (n_obs,) float64.
 
-    Returns (loss[B], grad[B, P]) (grad is None in value-only mode); with
-    magnitudes=True (reverse mode) also mag[B, P], the gradient propagated through
-    absolute values -- the size of the terms each component sums.  f32=True evaluates
+    Returns (loss[B], grad[B, P]) (grad is None in value-only mode).  f32=True evaluates
     in binary32 arithmetic (each result rounded to float; inputs rounded first).
     """
     lib = _load()
@@ -82,16 +80,13 @@ def run(program: str, params, obs, *, frontend: int = FRONTEND_SCHEME, mode: int
     B, P = params.shape
     loss = np.zeros(B, dtype=np.float64)
     grad = np.zeros((B, P), dtype=np.float64) if mode != MODE_VALUE else None
-    mag = np.zeros((B, P), dtype=np.float64) if (magnitudes and mode == MODE_REVERSE) else None
     err = ctypes.create_string_buffer(1024)
     text = program.encode()
     rc = lib.ndvm_oracle_run(text, len(text), frontend, B, P,
                              params.ctypes.data, obs.size, obs.ctypes.data if obs.size else None,
                              loss.ctypes.data, grad.ctypes.data if grad is not None else None,
-                             mag.ctypes.data if mag is not None else None, mode | (4 if f32 else 0), nthreads,
+                             mode | (4 if f32 else 0), nthreads,
                              err, len(err))
     if rc != 0:
         raise OracleError(err.value.decode(errors="replace"))
-    if magnitudes:
-        return loss, grad, mag
     return loss, grad

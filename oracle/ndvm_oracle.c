@@ -122,7 +122,6 @@ typedef struct Num {
   int mark;           /* depth-first-search state for the backward ordering */
   double* v;          /* primal values, row-major r*c */
   double* g;          /* adjoint, allocated in the backward pass */
-  double* gm;         /* magnitude adjoint: the same propagation on absolute values */
   double* d;          /* dual partials: d[e*P + k] = d v[e] / d theta_k (NULL = all zero) */
 } Num;
 
@@ -699,22 +698,17 @@ static Num* matfun_num(Ctx* cx, int kind, Num* a) {
 /* The reachable graph is ordered by an explicit-stack depth-first search     */
 /* from the loss; adjoints flow from the loss towards the parameters.         */
 /* ------------------------------------------------------------------------- */
-static double* gbuf_sel(Ctx* cx, Num* n, int absmode) {
-  double** slot = absmode ? &n->gm : &n->g;
-  if (!*slot) {
+static double* gbuf(Ctx* cx, Num* n) {
+  if (!n->g) {
     size_t m = (size_t)n->r * n->c;
-    *slot = (double*)arena_alloc(cx->ar, sizeof(double) * m);
-    if (!*slot) fail(cx, "out of memory");
-    memset(*slot, 0, sizeof(double) * m);
+    n->g = (double*)arena_alloc(cx->ar, sizeof(double) * m);
+    if (!n->g) fail(cx, "out of memory");
+    memset(n->g, 0, sizeof(double) * m);
   }
-  return *slot;
+  return n->g;
 }
 
-/* absmode = 1 runs the same propagation on absolute values (|g| times |local
- * derivative|, every contribution added): the result bounds the magnitude of the
- * terms summed into each gradient component, the scale against which rounding
- * in any summation order is measured. */
-static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
+static void backward(Ctx* cx, Num* loss, double* grad) {
   /* post-order over dependent nodes */
   size_t cap = 1024, cnt = 0, sp = 0;
   Num** order = (Num**)malloc(sizeof(Num*) * cap);
@@ -722,15 +716,15 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
   Num** stk = (Num**)malloc(sizeof(Num*) * scap);
   int* sidx = (int*)malloc(sizeof(int) * scap);
   if (!loss->dep) { free(order); free(stk); free(sidx); return; }
-  stk[0] = loss; sidx[0] = 0; sp = 1; loss->mark = absmode ? 3 : 1;
+  stk[0] = loss; sidx[0] = 0; sp = 1; loss->mark = 1;
   while (sp) {
     Num* n = stk[sp - 1];
     int i = sidx[sp - 1];
     if (i < n->nin) {
       sidx[sp - 1] = i + 1;
       Num* m = n->in[i];
-      if (m->dep && m->mark != (absmode ? 3 : 1)) {
-        m->mark = absmode ? 3 : 1;
+      if (m->dep && m->mark != 1) {
+        m->mark = 1;
         if (sp == scap) { scap *= 2; stk = (Num**)realloc(stk, sizeof(Num*) * scap); sidx = (int*)realloc(sidx, sizeof(int) * scap); }
         stk[sp] = m; sidx[sp] = 0; sp++;
       }
@@ -740,15 +734,13 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
     }
   }
   free(stk); free(sidx);
-  gbuf_sel(cx, loss, absmode)[0] = 1.0;
-#define gbuf(cx, x) gbuf_sel(cx, x, absmode)
-#define F(v) (absmode ? fabs(v) : (v))
-#define ADD(dst, v) ((dst) = RF(cx, (dst) + (absmode ? fabs(v) : RF(cx, (v)))))
-#define SUB(dst, v) ((dst) = RF(cx, (dst) + (absmode ? fabs(v) : -RF(cx, (v)))))
+  gbuf(cx, loss)[0] = 1.0;
+#define ADD(dst, v) ((dst) = RF(cx, (dst) + RF(cx, (v))))
+#define SUB(dst, v) ((dst) = RF(cx, (dst) + -RF(cx, (v))))
   for (size_t q = cnt; q-- > 0;) {
     Num* n = order[q];
     size_t m = (size_t)n->r * n->c;
-    double* g = absmode ? n->gm : n->g;
+    double* g = n->g;
     if (!g) continue;
     int nz = 0;
     for (size_t e = 0; e < m; e++) if (g[e] != 0.0) { nz = 1; break; }
@@ -770,7 +762,7 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
       case N_MUL:
         for (int i = 0; i < n->nin; i++) if (x[i]->dep) {
           double p = 1.0;
-          for (int j = 0; j < n->nin; j++) if (j != i) p *= F(x[j]->v[0]);
+          for (int j = 0; j < n->nin; j++) if (j != i) p *= x[j]->v[0];
           ADD(gbuf(cx, x[i])[0], g[0] * p);
         }
         break;
@@ -836,7 +828,7 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
         break;
       case N_MSCALE: {
         Num* s = x[0]; Num* a = x[1];
-        if (s->dep) { double t = 0; for (size_t e = 0; e < m; e++) t += g[e] * F(a->v[e]); ADD(gbuf(cx, s)[0], t); }
+        if (s->dep) { double t = 0; for (size_t e = 0; e < m; e++) t += g[e] * a->v[e]; ADD(gbuf(cx, s)[0], t); }
         if (a->dep) { double* ga = gbuf(cx, a); for (size_t e = 0; e < m; e++) ADD(ga[e], s->v[0] * g[e]); }
         break;
       }
@@ -847,14 +839,14 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
         if (A->dep) {
           double* ga = gbuf(cx, A);
           for (int i = 0; i < nr; i++) for (int k = 0; k < K; k++) {
-            double s = 0; for (int j = 0; j < nc; j++) s += g[i * nc + j] * F(B->v[k * nc + j]);
+            double s = 0; for (int j = 0; j < nc; j++) s += g[i * nc + j] * B->v[k * nc + j];
             ADD(ga[i * K + k], s);
           }
         }
         if (B->dep) {
           double* gb = gbuf(cx, B);
           for (int k = 0; k < K; k++) for (int j = 0; j < nc; j++) {
-            double s = 0; for (int i = 0; i < nr; i++) s += F(A->v[i * K + k]) * g[i * nc + j];
+            double s = 0; for (int i = 0; i < nr; i++) s += A->v[i * K + k] * g[i * nc + j];
             ADD(gb[k * nc + j], s);
           }
         }
@@ -876,7 +868,7 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
         int k = n->r; double* Bv = n->v; double* ga = gbuf(cx, x[0]);
         for (int i = 0; i < k; i++) for (int j = 0; j < k; j++) {
           double s = 0;
-          for (int p = 0; p < k; p++) for (int q2 = 0; q2 < k; q2++) s += F(Bv[p * k + i]) * g[p * k + q2] * F(Bv[j * k + q2]);
+          for (int p = 0; p < k; p++) for (int q2 = 0; q2 < k; q2++) s += Bv[p * k + i] * g[p * k + q2] * Bv[j * k + q2];
           SUB(ga[i * k + j], s);
         }
         break;
@@ -887,7 +879,7 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
         double* inv = (double*)malloc(sizeof(double) * k * k);
         double det;
         inv_det(k, x[0]->v, inv, &det);
-        double f = n->kind == N_DET ? g[0] * F(n->v[0]) : g[0];
+        double f = n->kind == N_DET ? g[0] * n->v[0] : g[0];
         double* ga = gbuf(cx, x[0]);
         for (int i = 0; i < k; i++) for (int j = 0; j < k; j++) ADD(ga[i * k + j], f * inv[j * k + i]);
         free(inv);
@@ -896,8 +888,6 @@ static void backward(Ctx* cx, Num* loss, double* grad, int absmode) {
       default: free(order); fail(cx, "internal: no adjoint rule for node kind %d", n->kind);
     }
   }
-#undef gbuf
-#undef F
 #undef ADD
 #undef SUB
   free(order);
@@ -1465,7 +1455,7 @@ static Num* run_bytecode(Ctx* cx) {
 typedef struct {
   const Program* prog; int frontend, mode, P;
   const double* params; const double* obs; long long nobs;
-  double* loss; double* grad; double* mag;
+  double* loss; double* grad;
   long long b0, b1;
   int status; char err[512];
   int f32;
@@ -1490,14 +1480,9 @@ static int run_lane(Job* jb, Arena* ar, long long b, double* g) {
   jb->loss[b] = loss->v[0];
   if (jb->grad && jb->mode != MODE_VALUE) {
     for (int k = 0; k < jb->P; k++) g[k] = 0.0;
-    if (jb->mode == MODE_REVERSE) backward(&cx, loss, g, 0);
+    if (jb->mode == MODE_REVERSE) backward(&cx, loss, g);
     else if (loss->d) for (int k = 0; k < jb->P; k++) g[k] = loss->d[k];
     for (int k = 0; k < jb->P; k++) jb->grad[b * jb->P + k] = g[k];
-    if (jb->mag && jb->mode == MODE_REVERSE) {
-      for (int k = 0; k < jb->P; k++) g[k] = 0.0;
-      backward(&cx, loss, g, 1);
-      for (int k = 0; k < jb->P; k++) jb->mag[b * jb->P + k] = g[k];
-    }
   }
   return OR_OK;
 }
@@ -1530,8 +1515,6 @@ static void free_program(Program* pg) {
  *   params      : B x P row-major parameters (host)
  *   obs/nobs    : observations shared by every lane (host)
  *   loss        : B outputs; grad: B x P outputs or NULL
- *   mag         : B x P magnitude scales (reverse mode only) or NULL: the gradient
- *                 propagated through absolute values, bounding the terms summed
  *   mode        : 0 value only, 1 reverse mode, 2 dual numbers; + 4 = fp32 mode
  *                 (every arithmetic result rounded to binary32; obs must be
  *                 given already rounded to float)
@@ -1540,7 +1523,7 @@ static void free_program(Program* pg) {
  */
 int ndvm_oracle_run(const char* program, size_t len, int frontend, long long B, int P,
                     const double* params, long long nobs, const double* obs,
-                    double* loss, double* grad, double* mag, int mode, int nthreads, char* err, size_t errcap) {
+                    double* loss, double* grad, int mode, int nthreads, char* err, size_t errcap) {
   Program pg; memset(&pg, 0, sizeof(pg));
   if (err && errcap) err[0] = 0;
   const int f32 = (mode & 4) != 0;
@@ -1573,7 +1556,7 @@ int ndvm_oracle_run(const char* program, size_t len, int frontend, long long B, 
   for (int t = 0; t < nthreads; t++) {
     Job* j = &jobs[t];
     j->prog = &pg; j->frontend = frontend; j->mode = mode; j->P = P; j->f32 = f32;
-    j->params = params; j->obs = obs; j->nobs = nobs; j->loss = loss; j->grad = grad; j->mag = mag;
+    j->params = params; j->obs = obs; j->nobs = nobs; j->loss = loss; j->grad = grad;
     j->b0 = t * per; j->b1 = (t + 1) * per < B ? (t + 1) * per : B;
     if (j->b0 > B) j->b0 = B;
   }
