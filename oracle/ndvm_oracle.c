@@ -474,7 +474,7 @@ static Num* dot_num(Ctx* cx, int n, Num** a, Num** b) {
   for (int i = 0; i < n; i++) { z->in[i] = a[i]; z->in[n + i] = b[i]; }
   z->ia = n; z->dep = any_dep(z);
   double s = 0;
-  for (int i = 0; i < n; i++) { double t = a[i]->v[0] * b[i]->v[0]; s = (i == 0) ? t : s + t; }
+  for (int i = 0; i < n; i++) { double t = RF(cx, a[i]->v[0] * b[i]->v[0]); s = (i == 0) ? t : RF(cx, s + t); }
   z->v[0] = s;
   if (cx->mode == MODE_DUAL && z->dep) {
     dual_alloc(cx, z);
@@ -535,7 +535,7 @@ static Num* madd_num(Ctx* cx, int kind, Num* a, Num* b) {
   Num* z = new_num(cx, kind, a->r, a->c, 2);
   z->in[0] = a; z->in[1] = b; z->dep = any_dep(z);
   int m = a->r * a->c;
-  for (int i = 0; i < m; i++) z->v[i] = kind == N_MADD ? a->v[i] + b->v[i] : a->v[i] - b->v[i];
+  for (int i = 0; i < m; i++) z->v[i] = RF(cx, kind == N_MADD ? a->v[i] + b->v[i] : a->v[i] - b->v[i]);
   if (cx->mode == MODE_DUAL && z->dep) {
     dual_alloc(cx, z);
     for (int i = 0; i < m; i++) for (int k = 0; k < cx->P; k++) {
@@ -550,7 +550,7 @@ static Num* mscale_num(Ctx* cx, Num* s, Num* a) {
   Num* z = new_num(cx, N_MSCALE, a->r, a->c, 2);
   z->in[0] = s; z->in[1] = a; z->dep = any_dep(z);
   int m = a->r * a->c;
-  for (int i = 0; i < m; i++) z->v[i] = s->v[0] * a->v[i];
+  for (int i = 0; i < m; i++) z->v[i] = RF(cx, s->v[0] * a->v[i]);
   if (cx->mode == MODE_DUAL && z->dep) {
     dual_alloc(cx, z);
     for (int i = 0; i < m; i++) for (int k = 0; k < cx->P; k++)
@@ -565,7 +565,7 @@ static Num* matmul_num(Ctx* cx, Num* a, Num* b) {
   int n = a->r, K = a->c, m = b->c;
   for (int i = 0; i < n; i++) for (int j = 0; j < m; j++) {
     double s = 0;
-    for (int k = 0; k < K; k++) { double t = a->v[i * K + k] * b->v[k * m + j]; s = (k == 0) ? t : s + t; }
+    for (int k = 0; k < K; k++) { double t = RF(cx, a->v[i * K + k] * b->v[k * m + j]); s = (k == 0) ? t : RF(cx, s + t); }
     z->v[i * m + j] = s;
   }
   if (cx->mode == MODE_DUAL && z->dep) {
@@ -592,31 +592,32 @@ static Num* transpose_num(Ctx* cx, Num* a) {
 
 /* Inverse and determinant of an n x n matrix (R4): closed-form adjugate for n <= 3,
  * Gauss-Jordan elimination with partial pivoting otherwise. */
-static void inv_det(int n, const double* a, double* inv, double* det) {
-  if (n == 1) { *det = a[0]; inv[0] = 1.0 / a[0]; return; }
+static void inv_det(Ctx* cx, int n, const double* a, double* inv, double* det) {
+#define R(x) RF(cx, (x))
+  if (n == 1) { *det = a[0]; inv[0] = R(1.0 / a[0]); return; }
   if (n == 2) {
-    double d = a[0] * a[3] - a[1] * a[2];
+    double d = R(R(a[0] * a[3]) - R(a[1] * a[2]));
     *det = d;
-    inv[0] = a[3] / d; inv[1] = -a[1] / d; inv[2] = -a[2] / d; inv[3] = a[0] / d;
+    inv[0] = R(a[3] / d); inv[1] = R(-a[1] / d); inv[2] = R(-a[2] / d); inv[3] = R(a[0] / d);
     return;
   }
   if (n == 3) {
     /* cofactors C_ij of A */
-    double c00 = a[4] * a[8] - a[5] * a[7];
-    double c01 = a[5] * a[6] - a[3] * a[8];
-    double c02 = a[3] * a[7] - a[4] * a[6];
-    double c10 = a[2] * a[7] - a[1] * a[8];
-    double c11 = a[0] * a[8] - a[2] * a[6];
-    double c12 = a[1] * a[6] - a[0] * a[7];
-    double c20 = a[1] * a[5] - a[2] * a[4];
-    double c21 = a[2] * a[3] - a[0] * a[5];
-    double c22 = a[0] * a[4] - a[1] * a[3];
-    double d = a[0] * c00 + a[1] * c01 + a[2] * c02;
+    double c00 = R(R(a[4] * a[8]) - R(a[5] * a[7]));
+    double c01 = R(R(a[5] * a[6]) - R(a[3] * a[8]));
+    double c02 = R(R(a[3] * a[7]) - R(a[4] * a[6]));
+    double c10 = R(R(a[2] * a[7]) - R(a[1] * a[8]));
+    double c11 = R(R(a[0] * a[8]) - R(a[2] * a[6]));
+    double c12 = R(R(a[1] * a[6]) - R(a[0] * a[7]));
+    double c20 = R(R(a[1] * a[5]) - R(a[2] * a[4]));
+    double c21 = R(R(a[2] * a[3]) - R(a[0] * a[5]));
+    double c22 = R(R(a[0] * a[4]) - R(a[1] * a[3]));
+    double d = R(R(R(a[0] * c00) + R(a[1] * c01)) + R(a[2] * c02));
     *det = d;
     /* inverse = transpose of the cofactor matrix / det */
-    inv[0] = c00 / d; inv[1] = c10 / d; inv[2] = c20 / d;
-    inv[3] = c01 / d; inv[4] = c11 / d; inv[5] = c21 / d;
-    inv[6] = c02 / d; inv[7] = c12 / d; inv[8] = c22 / d;
+    inv[0] = R(c00 / d); inv[1] = R(c10 / d); inv[2] = R(c20 / d);
+    inv[3] = R(c01 / d); inv[4] = R(c11 / d); inv[5] = R(c21 / d);
+    inv[6] = R(c02 / d); inv[7] = R(c12 / d); inv[8] = R(c22 / d);
     return;
   }
   /* Gauss-Jordan on [A | I] */
@@ -632,16 +633,17 @@ static void inv_det(int n, const double* a, double* inv, double* det) {
       d = -d;
     }
     double p = w[col * 2 * n + col];
-    d *= p;
-    for (int j = 0; j < 2 * n; j++) w[col * 2 * n + j] /= p;
+    d = R(d * p);
+    for (int j = 0; j < 2 * n; j++) w[col * 2 * n + j] = R(w[col * 2 * n + j] / p);
     for (int i = 0; i < n; i++) if (i != col) {
       double f = w[i * 2 * n + col];
-      if (f != 0) for (int j = 0; j < 2 * n; j++) w[i * 2 * n + j] -= f * w[col * 2 * n + j];
+      if (f != 0) for (int j = 0; j < 2 * n; j++) w[i * 2 * n + j] = R(w[i * 2 * n + j] - R(f * w[col * 2 * n + j]));
     }
   }
   for (int i = 0; i < n; i++) for (int j = 0; j < n; j++) inv[i * n + j] = w[i * 2 * n + n + j];
   *det = d;
   free(w);
+#undef R
 }
 
 static Num* matfun_num(Ctx* cx, int kind, Num* a) {
@@ -650,7 +652,7 @@ static Num* matfun_num(Ctx* cx, int kind, Num* a) {
   if (kind == N_TRACE) {
     Num* z = new_num(cx, N_TRACE, 1, 1, 1);
     z->in[0] = a; z->dep = a->dep;
-    double s = 0; for (int i = 0; i < n; i++) s = (i == 0) ? a->v[0] : s + a->v[i * n + i];
+    double s = 0; for (int i = 0; i < n; i++) s = (i == 0) ? a->v[0] : RF(cx, s + a->v[i * n + i]);
     z->v[0] = s;
     if (cx->mode == MODE_DUAL && a->d) {
       dual_alloc(cx, z);
@@ -660,14 +662,14 @@ static Num* matfun_num(Ctx* cx, int kind, Num* a) {
   }
   double* inv = (double*)arena_alloc(cx->ar, sizeof(double) * n * n);
   double det;
-  inv_det(n, a->v, inv, &det);
+  inv_det(cx, n, a->v, inv, &det);
   Num* z;
   if (kind == N_INV) {
     z = new_num(cx, N_INV, n, n, 1);
     memcpy(z->v, inv, sizeof(double) * n * n);
   } else {
     z = new_num(cx, kind, 1, 1, 1);
-    z->v[0] = kind == N_DET ? det : log(det);
+    z->v[0] = kind == N_DET ? det : RF(cx, log(det));
   }
   z->in[0] = a; z->dep = a->dep;
   if (cx->mode == MODE_DUAL && a->d) {
@@ -828,7 +830,7 @@ static void backward(Ctx* cx, Num* loss, double* grad) {
         break;
       case N_MSCALE: {
         Num* s = x[0]; Num* a = x[1];
-        if (s->dep) { double t = 0; for (size_t e = 0; e < m; e++) t += g[e] * a->v[e]; ADD(gbuf(cx, s)[0], t); }
+        if (s->dep) { double t = 0; for (size_t e = 0; e < m; e++) t = RF(cx, t + RF(cx, g[e] * a->v[e])); ADD(gbuf(cx, s)[0], t); }
         if (a->dep) { double* ga = gbuf(cx, a); for (size_t e = 0; e < m; e++) ADD(ga[e], s->v[0] * g[e]); }
         break;
       }
@@ -839,14 +841,14 @@ static void backward(Ctx* cx, Num* loss, double* grad) {
         if (A->dep) {
           double* ga = gbuf(cx, A);
           for (int i = 0; i < nr; i++) for (int k = 0; k < K; k++) {
-            double s = 0; for (int j = 0; j < nc; j++) s += g[i * nc + j] * B->v[k * nc + j];
+            double s = 0; for (int j = 0; j < nc; j++) s = RF(cx, s + RF(cx, g[i * nc + j] * B->v[k * nc + j]));
             ADD(ga[i * K + k], s);
           }
         }
         if (B->dep) {
           double* gb = gbuf(cx, B);
           for (int k = 0; k < K; k++) for (int j = 0; j < nc; j++) {
-            double s = 0; for (int i = 0; i < nr; i++) s += A->v[i * K + k] * g[i * nc + j];
+            double s = 0; for (int i = 0; i < nr; i++) s = RF(cx, s + RF(cx, A->v[i * K + k] * g[i * nc + j]));
             ADD(gb[k * nc + j], s);
           }
         }
@@ -868,7 +870,8 @@ static void backward(Ctx* cx, Num* loss, double* grad) {
         int k = n->r; double* Bv = n->v; double* ga = gbuf(cx, x[0]);
         for (int i = 0; i < k; i++) for (int j = 0; j < k; j++) {
           double s = 0;
-          for (int p = 0; p < k; p++) for (int q2 = 0; q2 < k; q2++) s += Bv[p * k + i] * g[p * k + q2] * Bv[j * k + q2];
+          for (int p = 0; p < k; p++) for (int q2 = 0; q2 < k; q2++)
+            s = RF(cx, s + RF(cx, RF(cx, Bv[p * k + i] * g[p * k + q2]) * Bv[j * k + q2]));
           SUB(ga[i * k + j], s);
         }
         break;
@@ -878,8 +881,8 @@ static void backward(Ctx* cx, Num* loss, double* grad) {
         int k = x[0]->r;
         double* inv = (double*)malloc(sizeof(double) * k * k);
         double det;
-        inv_det(k, x[0]->v, inv, &det);
-        double f = n->kind == N_DET ? g[0] * n->v[0] : g[0];
+        inv_det(cx, k, x[0]->v, inv, &det);
+        double f = n->kind == N_DET ? RF(cx, g[0] * n->v[0]) : g[0];
         double* ga = gbuf(cx, x[0]);
         for (int i = 0; i < k; i++) for (int j = 0; j < k; j++) ADD(ga[i * k + j], f * inv[j * k + i]);
         free(inv);
