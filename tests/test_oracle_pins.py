@@ -167,6 +167,68 @@ def test_kalman_rand8_is_dense_gaussian(oracle_mod):
         assert_rel(grad[b], g, 1e-8, scale=np.max(np.abs(g)))
 
 
+@pytest.mark.parametrize("m", [4, 6, 8])
+def test_kalman_highd_is_dense_gaussian(oracle_mod, m):
+    """The population Kalman likelihood with an m x m innovation covariance (m = 4..8,
+    the elimination branch of the oracle's determinant, log-determinant and inverse)
+    equals the dense Gaussian NLL of the stacked observations, and its gradient the
+    trace formula (Appendix C's logdet and inv adjoints, prediction-error decomposition)."""
+    T, D = 3, 12
+    w = W.kalman_highd(B=3, D=D, m=m, T=T)
+    F = w.meta["F"]
+    H = np.zeros((m, D))
+    H[:, :m] = np.eye(m)
+    y = w.obs[: m * T]
+    loss, grad = run(oracle_mod, w.program, w.params, y)
+
+    def sig(v):
+        return lgssm_dense_cov(F, H, v[0] * np.eye(D), v[1] * np.eye(m), v[2] * np.eye(D), T)
+
+    base = sig(np.zeros(3))
+    A = [sig(np.eye(3)[k]) - base for k in range(3)]
+    for b in range(w.B):
+        v = np.exp(2 * w.params[b])
+        Sig = base + sum(v[k] * A[k] for k in range(3))
+        nll, g = dense_gaussian_nll(y, Sig, [2 * v[k] * A[k] for k in range(3)])
+        assert_rel(loss[b], nll, 1e-11)
+        assert_rel(grad[b], g, 1e-9, scale=np.max(np.abs(g)))
+
+
+@pytest.mark.parametrize("n", [4, 5, 6, 8])
+def test_det_logdet_by_elimination_against_lapack(oracle_mod, n):
+    """det and logdet of non-symmetric n x n matrices (n >= 4: the oracle eliminates with
+    partial pivoting) against LAPACK's LU determinant. The matrices are row permutations
+    of diagonally dominant ones, so every column's pivot lies below the diagonal and the
+    elimination swaps rows; an odd permutation makes det negative. Gradients follow
+    Appendix C: d det/dA = det(A) A^-T, d logdet/dA = A^-T."""
+    rng = np.random.default_rng(100 + n)
+    names = " ".join(f"p{k}" for k in range(n * n))
+    DET = f"(model (params {names}) (det (matrix {n} {n} {names})))"
+    LOGDET = f"(model (params {names}) (logdet (matrix {n} {n} {names})))"
+    for trial in range(3):
+        base = rng.normal(0, 0.6, (n, n)) + np.diag(rng.uniform(2.0, 4.0, n) * rng.choice([-1.0, 1.0], n))
+        perm = np.roll(np.arange(n), 1 + trial)          # a cyclic shift: every pivot is off the diagonal
+        A = base[perm]
+        assert not np.array_equal(perm, np.arange(n))
+        l, g = run(oracle_mod, DET, A.reshape(1, -1))
+        d = np.linalg.det(A)
+        assert_rel(l[0], d, 1e-12)
+        np.testing.assert_allclose(g[0].reshape(n, n), d * np.linalg.inv(A).T, rtol=1e-11,
+                                   atol=1e-12 * abs(d) * np.max(np.abs(np.linalg.inv(A))))
+        Ap = A if d > 0 else A[np.r_[1, 0, 2:n]]         # one more swap makes det positive
+        sgn, ld = np.linalg.slogdet(Ap)
+        assert sgn > 0
+        l2, g2 = run(oracle_mod, LOGDET, Ap.reshape(1, -1))
+        assert abs(l2[0] - ld) <= 1e-13 * max(1.0, abs(ld))
+        np.testing.assert_allclose(g2[0].reshape(n, n), np.linalg.inv(Ap).T, rtol=1e-11,
+                                   atol=1e-12 * np.max(np.abs(np.linalg.inv(Ap))))
+    # the sign of an odd permutation of a positive-determinant matrix
+    M = np.eye(n) * 3.0 + rng.normal(0, 0.3, (n, n))
+    odd = M[np.r_[1, 0, 2:n]]
+    l, _ = run(oracle_mod, DET, odd.reshape(1, -1))
+    assert np.sign(l[0]) == np.sign(np.linalg.det(odd)) == -np.sign(np.linalg.det(M))
+
+
 # --------------------------------------------------- logistic: tangent-linear recursion
 def test_logistic_forward_sensitivity(oracle_mod):
     w = W.logistic(B=6)
@@ -363,29 +425,60 @@ def test_reverse_mode_equals_dual_numbers(oracle_mod, cfg):
 @pytest.mark.parametrize("case", ["cv4_T200", "rand8_T1000", "highd_D12"])
 def test_parity_rule_rejects_perturbed_gradients(oracle_mod, case):
     """The 1e-12 comparison rule measures each gradient component against the lane's
-    largest oracle component only, so on the Kalman likelihoods -- whose recursions make
-    the terms summed into a component many orders larger than the component -- it still
-    rejects a sign-flipped gradient, one perturbed by 1e-9 relative and a loss perturbed
-    by 1e-11, while it accepts the oracle's dual-number gradient (a second derivative
-    engine with another summation order: the rounding spread the tolerance must admit)."""
-    from conftest import rel_check
+    largest oracle component, so on the Kalman likelihoods -- whose recursions make the
+    terms summed into a component many orders larger than the component -- it still
+    rejects a sign-flipped gradient, one perturbed by 1e-9 relative, a dropped component
+    and a loss perturbed by 1e-11, while it accepts the oracle's dual-number gradient (a
+    second derivative engine with another summation order).  The measured rounding
+    spread of every Kalman lane is below 1e-13, so no lane's bound is relaxed."""
+    from conftest import oracle_ref, rel_check
     w = {"cv4_T200": lambda: W.kalman_cv4(B=6, T=200), "rand8_T1000": lambda: W.kalman_rand8(B=3),
          "highd_D12": lambda: W.kalman_highd(B=3, D=12, m=4, T=6)}[case]()
-    l, g = oracle_mod.run(w.program, w.params, w.obs, nthreads=6)
+    l, g, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs, nthreads=6)
+    assert sp.max() < 1e-13, sp
     ld, gd = oracle_mod.run(w.program, w.params, w.obs, nthreads=6, mode=oracle_mod.MODE_DUAL)
-    ok, rep = rel_check(ld, gd, l, g, 1e-12)
-    assert ok and rep["worst_grad"] < 1e-13, rep
-    assert not rel_check(l, -g, l, g, 1e-12)[0]
+    ok, rep = rel_check(ld, gd, l, g, 1e-12, sp)
+    assert ok and rep["relaxed_lanes"] == 0, rep
+    assert not rel_check(l, -g, l, g, 1e-12, sp)[0]
     rng = np.random.default_rng(0)
-    assert not rel_check(l, g * (1 + 1e-9 * rng.choice([-1.0, 1.0], g.shape)), l, g, 1e-12)[0]
+    assert not rel_check(l, g * (1 + 1e-9 * rng.choice([-1.0, 1.0], g.shape)), l, g, 1e-12, sp)[0]
     k = int(np.argmax(np.abs(g[0])))
     g1 = g.copy()
     g1[0, k] *= 1 + 1e-9
-    assert not rel_check(l, g1, l, g, 1e-12)[0]
-    assert not rel_check(l * (1 + 1e-11), g, l, g, 1e-12)[0]
+    assert not rel_check(l, g1, l, g, 1e-12, sp)[0]
+    assert not rel_check(l * (1 + 1e-11), g, l, g, 1e-12, sp)[0]
     g2 = g.copy()
     g2[:, 0] = 0.0          # a dropped component
-    assert not rel_check(l, g2, l, g, 1e-12)[0]
+    assert not rel_check(l, g2, l, g, 1e-12, sp)[0]
+
+
+def test_ill_conditioned_lane_spread(oracle_mod):
+    """Lane 12 of random program 27 (200-program set, seed 1234, 37 lanes): its only
+    parameter t0 = -0.0041 enters through log|1 + t0^2| and nested g / (1 + g^2) terms,
+    whose derivative 1/(1 + g^2) - 2 g^2 / (1 + g^2)^2 cancels near g = 1; the gradient is
+    4.5e-12 while its per-point contributions are 140 times larger and cancel too.  The
+    oracle's reverse mode and dual numbers disagree there by about 2e-10 of the gradient,
+    so no evaluation order can be checked at 1e-12: the rule relaxes this lane to 8 times
+    that spread, which still rejects a sign flip or a 1e-8 perturbation.  Such lanes are
+    rare: 15 of the 7400 lanes of all 200 programs (12 of them in program 27, whose
+    parameter only enters through log|1 + t0^2| with t0 near 0); the test allows 1 %."""
+    from conftest import oracle_ref, rel_check
+    ws = W.random_exprs(n_programs=200, B=37, n_points=256, seed=1234)
+    w = ws[27]
+    l, g, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs)
+    assert sp[12] > 1e-11 and np.abs(g[12]).max() < 1e-10, (sp[12], g[12])
+    ok, rep = rel_check(l, g * (1 + 1e-13), l, g, 1e-12, sp)
+    assert ok and rep["relaxed_lanes"] >= 1, rep
+    assert not rel_check(l, -g, l, g, 1e-12, sp)[0]
+    g1 = g.copy()
+    g1[12] *= 1 + 1e-8
+    assert not rel_check(l, g1, l, g, 1e-12, sp)[0]
+    relaxed = total = 0
+    for v in ws:
+        _, _, s = oracle_ref(oracle_mod, v.program, v.params, v.obs)
+        relaxed += int((8 * s > 1e-12).sum())
+        total += len(s)
+    assert relaxed <= total // 100, (relaxed, total)
 
 
 def test_threads_do_not_change_results(oracle_mod):
@@ -450,6 +543,41 @@ def test_fp32_mode_is_binary32_arithmetic(oracle_mod):
     l, g = oracle_mod.run(bc, np.array([[0.1]]), np.array([0.2]), frontend=1, f32=True)
     assert l[0] == float((f(0.1) + f(0.2)) * f(0.3))
     assert g[0, 0] == float(f(0.3))
+
+
+def test_fp32_mode_matrix_primitives_are_binary32(oracle_mod):
+    """Matrix primitives in fp32 mode round every product and every partial sum to
+    binary32 (IEEE 754 single precision), as the fp32 variant's arithmetic does.  A dot
+    product 1 + 2^-24 + 2^-24 accumulated in binary32 stays 1 (each addition is a tie
+    rounded to even), whereas accumulating in binary64 and rounding once gives 1 + 2^-23;
+    the same for a matrix product, a trace, a matrix sum, and the pivot products of the
+    elimination that gives a 4 x 4 determinant."""
+    e = 2.0 ** -24
+    for prog in ("(model (params a b c) (dot (matrix 3 1 a b c) (matrix 3 1 1.0 1.0 1.0)))",
+                 "(model (params a b c) (mref (matmul (matrix 1 3 a b c) (matrix 3 1 1.0 1.0 1.0)) 0 0))",
+                 "(model (params a b c) (trace (matrix 3 3 a 0.0 0.0 0.0 b 0.0 0.0 0.0 c)))"):
+        l32, _ = oracle_mod.run(prog, np.array([[1.0, e, e]]), np.zeros(0), f32=True)
+        l64, _ = oracle_mod.run(prog, np.array([[1.0, e, e]]), np.zeros(0))
+        assert l32[0] == 1.0 and l64[0] == 1.0 + 2 * e, prog
+    # matrix sum: (1 + 2^-24) is not a binary32 value; the element rounds to 1
+    l32, _ = oracle_mod.run("(model (params a b) (mref (m+ (matrix 1 1 a) (matrix 1 1 b)) 0 0))",
+                            np.array([[1.0, e]]), np.zeros(0), f32=True)
+    assert l32[0] == 1.0
+    # 4 x 4 determinant (elimination): every output is a binary32 value, within a few
+    # binary32 ulps of LAPACK's binary64 value, and not the binary64 value rounded once
+    rng = np.random.default_rng(4)
+    names = " ".join(f"p{k}" for k in range(16))
+    DET = f"(model (params {names}) (det (matrix 4 4 {names})))"
+    diffs = 0
+    for _ in range(20):
+        A = (rng.normal(0, 1, (4, 4)) + 3 * np.eye(4)).astype(np.float32).astype(np.float64)
+        l32, g32 = oracle_mod.run(DET, A.reshape(1, -1), np.zeros(0), f32=True)
+        assert float(np.float32(l32[0])) == l32[0]
+        assert np.all(g32.astype(np.float32).astype(np.float64) == g32)
+        d = np.linalg.det(A)
+        assert abs(l32[0] - d) <= 64 * np.finfo(np.float32).eps * abs(d)
+        diffs += l32[0] != float(np.float32(d))
+    assert diffs > 0
 
 
 def test_control_fuzz_reverse_equals_dual_numbers_and_fd(oracle_mod):
