@@ -45,15 +45,43 @@ def cuda():
     return torch.device("cuda:0")
 
 
-def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol):
+# A lane's bound is relaxed only where the oracle's own two derivative engines disagree
+# by more than tol / SPREAD_FACTOR; there it is SPREAD_FACTOR times their disagreement.
+SPREAD_FACTOR = 8.0
+
+
+def oracle_ref(oracle_mod, program, params, obs, frontend=0, f32=False, nthreads=8):
+    """The oracle's (loss, grad, spread) for every lane.
+
+    spread[b] = max_k |g_bk(reverse mode) - g_bk(dual numbers)| / max_j |g_bj(reverse)|:
+    the disagreement of the oracle's two independent derivative engines (the pointer-graph
+    reverse sweep and forward-mode dual numbers sum the same chain-rule terms in different
+    orders), a measured rounding spread of that lane's gradient.  It is about 1e-16..1e-14
+    on well-conditioned lanes (every Kalman lane included); it is large only where a
+    gradient is a near-total cancellation, where no two evaluation orders agree to 1e-12."""
+    loss, grad = oracle_mod.run(program, params, obs, frontend=frontend, nthreads=nthreads, f32=f32)
+    _, dual = oracle_mod.run(program, params, obs, frontend=frontend, nthreads=nthreads, f32=f32,
+                             mode=oracle_mod.MODE_DUAL)
+    if grad.size == 0:
+        return loss, grad, np.zeros(len(loss))
+    with np.errstate(invalid="ignore", divide="ignore"):
+        s = np.maximum(np.max(np.abs(grad), axis=1), 1e-300)
+        spread = np.max(np.abs(grad - dual), axis=1) / s
+    spread[~np.isfinite(spread)] = 0.0
+    return loss, grad, spread
+
+
+def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol, spread=None):
     """Comparison rule for one batch of lanes.
 
     Loss: |gpu - ora| <= tol * |ora|.  Gradient component k of lane b:
-    |gpu_bk - ora_bk| <= tol * max_j |ora_bj| -- the scale is the lane's largest oracle
+    |gpu_bk - ora_bk| <= tol_b * max_j |ora_bj| -- the scale is the lane's largest oracle
     gradient component, nothing else, so a sign-flipped or a 1e-9-perturbed gradient
-    fails.  A lane whose oracle loss is non-finite must be non-finite in the same class
-    (NaN vs +-inf) on the GPU and is excluded from the relative checks.
-    Returns (ok, report).
+    fails.  tol_b = max(tol, SPREAD_FACTOR * spread_b) with spread_b the lane's measured
+    rounding spread (oracle_ref); tol_b = tol when no spread is given.  The report counts
+    the lanes whose bound was relaxed.  A lane whose oracle loss is non-finite must be
+    non-finite in the same class (NaN vs +-inf) on the GPU and is excluded from the
+    relative checks.  Returns (ok, report).
     """
     gpu_loss = np.asarray(gpu_loss, dtype=np.float64)
     ora_loss = np.asarray(ora_loss, dtype=np.float64)
@@ -69,22 +97,30 @@ def rel_check(gpu_loss, gpu_grad, ora_loss, ora_grad, tol):
     if worst_l > tol:
         b = np.nonzero(fin)[0][int(np.argmax(el))]
         bad.append(f"loss lane {b}: gpu {gpu_loss[b]!r} oracle {ora_loss[b]!r} rel {worst_l:.3e}")
-    worst_g = 0.0
+    worst_g, relaxed, max_spread = 0.0, 0, 0.0
     if gpu_grad is not None and ora_grad is not None and ora_grad.size:
         g = np.asarray(gpu_grad, dtype=np.float64)[fin]
         o = np.asarray(ora_grad, dtype=np.float64)[fin]
         gfin = np.isfinite(o).all(axis=1)
         s = np.maximum(np.max(np.abs(o[gfin]), axis=1, keepdims=True), 1e-300)
+        lane_tol = np.full((int(gfin.sum()), 1), float(tol))
+        if spread is not None:
+            sp = np.asarray(spread, dtype=np.float64)[fin][gfin].reshape(-1, 1)
+            lane_tol = np.maximum(lane_tol, SPREAD_FACTOR * sp)
+            relaxed = int((lane_tol > tol).sum())
+            max_spread = float(sp.max()) if sp.size else 0.0
         eg = np.abs(g[gfin] - o[gfin]) / s
         worst_g = float(eg.max()) if eg.size else 0.0
-        if worst_g > tol:
-            i, k = np.unravel_index(int(np.argmax(eg)), eg.shape)
-            bad.append(f"grad lane {i} comp {k}: gpu {g[gfin][i, k]!r} oracle {o[gfin][i, k]!r} rel {worst_g:.3e}")
+        over = eg / lane_tol
+        if over.size and over.max() > 1.0:
+            i, k = np.unravel_index(int(np.argmax(over)), over.shape)
+            bad.append(f"grad lane {i} comp {k}: gpu {g[gfin][i, k]!r} oracle {o[gfin][i, k]!r} "
+                       f"rel {eg[i, k]:.3e} bound {lane_tol[i, 0]:.3e}")
         nf = ~gfin
         if nf.any() and not np.array_equal(np.isnan(g[nf]), np.isnan(o[nf])):
             bad.append("non-finite gradient class mismatch")
     return (not bad), {"worst_loss": worst_l, "worst_grad": worst_g, "nonfinite_lanes": int((~fin).sum()),
-                       "problems": bad}
+                       "relaxed_lanes": relaxed, "max_spread": max_spread, "problems": bad}
 
 
 # hand-derived fixtures under tests/golden (each cites the rule it exercises and shows

@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import rel_check
+from conftest import oracle_ref, rel_check
 
 pytestmark = pytest.mark.gpu
 
@@ -28,8 +28,8 @@ def test_fuzz_program_matches_oracle(ndvm, oracle_mod, cuda, k):
     w = PROGRAMS[k]
     tape = ndvm.trace_build(w.program, w.frontend)
     gl, gg = _gpu(ndvm, tape, w.params, w.obs)
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, frontend=w.frontend, nthreads=8)
-    ok, rep = rel_check(gl, gg, ol, og, 1e-12)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend)
+    ok, rep = rel_check(gl, gg, ol, og, 1e-12, sp)
     assert ok, rep
 
 

@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import rel_check
+from conftest import oracle_ref, rel_check
 
 pytestmark = pytest.mark.gpu
 
@@ -28,8 +28,8 @@ def _gpu(nd, w, lanes=None):
 def test_highd_kalman_matches_oracle(ndvm, oracle_mod, cuda, D, m, T):
     w = W.kalman_highd(B=20, D=D, m=m, T=T)
     gl, gg, fl = _gpu(ndvm, w)
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, nthreads=8)
-    ok, rep = rel_check(gl, gg, ol, og, 1e-12)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs)
+    ok, rep = rel_check(gl, gg, ol, og, 1e-12, sp)
     assert ok, rep
     np.testing.assert_array_equal(fl, gl)
 
@@ -40,8 +40,8 @@ def test_highd_kalman_full_size_sampled(ndvm, oracle_mod, cuda):
     w = W.kalman_highd()
     gl, gg, _ = _gpu(ndvm, w)
     idx = np.array([0, 341, 682, 1023])
-    ol, og = oracle_mod.run(w.program, w.params[idx], w.obs, nthreads=4)
-    ok, rep = rel_check(gl[idx], gg[idx], ol, og, 1e-12)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params[idx], w.obs, nthreads=4)
+    ok, rep = rel_check(gl[idx], gg[idx], ol, og, 1e-12, sp)
     assert ok, rep
 
 
@@ -74,6 +74,6 @@ def test_highd_fp32_variant(ndvm, oracle_mod, cuda):
     o = torch.tensor(w.obs, dtype=torch.float32, device="cuda")
     gl, gg = ndvm.value_and_grad(tape, p, o)
     torch.cuda.synchronize()
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, nthreads=8, f32=True)
-    ok, rep = rel_check(gl.double().cpu().numpy(), gg.double().cpu().numpy(), ol, og, 1e-5)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs, f32=True)
+    ok, rep = rel_check(gl.double().cpu().numpy(), gg.double().cpu().numpy(), ol, og, 1e-5, sp)
     assert ok, rep

@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import golden_cases, golden_close, hazard_workloads, load_golden, rel_check
+from conftest import golden_cases, golden_close, hazard_workloads, load_golden, oracle_ref, rel_check
 
 pytestmark = pytest.mark.gpu
 
@@ -31,14 +31,14 @@ def gpu_run(nd, w, dtype="f64", ws_bytes=None, lanes=None):
     return loss.double().cpu().numpy(), grad.double().cpu().numpy(), fl.double().cpu().numpy()
 
 
-def oracle_run(oracle_mod, w, idx=None, nthreads=8):
-    """(loss, grad) of the oracle for all lanes or the lanes idx."""
+def oracle_run(oracle_mod, w, idx=None, nthreads=8, f32=False):
+    """(loss, grad, spread) of the oracle for all lanes or the lanes idx (conftest.oracle_ref)."""
     params = w.params if idx is None else w.params[idx]
-    return oracle_mod.run(w.program, params, w.obs, frontend=w.frontend, nthreads=nthreads)
+    return oracle_ref(oracle_mod, w.program, params, w.obs, frontend=w.frontend, nthreads=nthreads, f32=f32)
 
 
-def check(gl, gg, ol, og, tol=TOL64):
-    ok, rep = rel_check(gl, gg, ol, og, tol)
+def check(gl, gg, ol, og, sp, tol=TOL64):
+    ok, rep = rel_check(gl, gg, ol, og, tol, sp)
     assert ok, rep
     return rep
 
@@ -46,8 +46,8 @@ def check(gl, gg, ol, og, tol=TOL64):
 def test_exp_decay_full(ndvm, oracle_mod, cuda):
     w = W.exp_decay()                      # B = 64 lanes, 50 points
     gl, gg, fl = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(fl, gl)  # value-only plan gives the same bits
 
 
@@ -55,8 +55,8 @@ def test_exp_decay_full(ndvm, oracle_mod, cuda):
 def test_exp_decay_ragged(ndvm, oracle_mod, cuda, B):
     w = W.exp_decay(B=B, n_points=23, seed=7)
     gl, gg, _ = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
 
 
 def test_random_exprs_small(ndvm, oracle_mod, cuda):
@@ -64,8 +64,8 @@ def test_random_exprs_small(ndvm, oracle_mod, cuda):
     worst = 0.0
     for w in ws:
         gl, gg, fl = gpu_run(ndvm, w)
-        ol, og = oracle_run(oracle_mod, w)
-        rep = check(gl, gg, ol, og)
+        ol, og, sp = oracle_run(oracle_mod, w)
+        rep = check(gl, gg, ol, og, sp)
         worst = max(worst, rep["worst_loss"], rep["worst_grad"])
         np.testing.assert_array_equal(fl, gl)
     print("worst relative error", worst)
@@ -78,15 +78,15 @@ def test_random_exprs_full_size_sampled(ndvm, oracle_mod, cuda):
     for w in ws:
         gl, gg, _ = gpu_run(ndvm, w)
         idx = np.sort(rng.choice(w.B, 64, replace=False))
-        ol, og = oracle_run(oracle_mod, w, idx)
-        check(gl[idx], gg[idx], ol, og)
+        ol, og, sp = oracle_run(oracle_mod, w, idx)
+        check(gl[idx], gg[idx], ol, og, sp)
 
 
 def test_logistic_bytecode(ndvm, oracle_mod, cuda):
     w = W.logistic(B=200)
     gl, gg, fl = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(fl, gl)
 
 
@@ -94,8 +94,8 @@ def test_logistic_full_size_sampled(ndvm, oracle_mod, cuda):
     w = W.logistic()                       # B = 16384
     gl, gg, _ = gpu_run(ndvm, w)
     idx = np.sort(np.random.default_rng(1).choice(w.B, 96, replace=False))
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(gl[idx], gg[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, sp)
 
 
 def test_logistic_workspace_chunks(ndvm, oracle_mod, cuda):
@@ -104,15 +104,15 @@ def test_logistic_workspace_chunks(ndvm, oracle_mod, cuda):
     tape = ndvm.trace_build(w.program, w.frontend)
     per_lane = tape.workspace_bytes(1)
     gl, gg, _ = gpu_run(ndvm, w, ws_bytes=per_lane * 300)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
 
 
 def test_kalman_cv4(ndvm, oracle_mod, cuda):
     w = W.kalman_cv4(B=70, T=200)
     gl, gg, fl = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(fl, gl)
 
 
@@ -120,15 +120,15 @@ def test_kalman_cv4_full_size_sampled(ndvm, oracle_mod, cuda):
     w = W.kalman_cv4()                     # B = 8192, T = 200
     gl, gg, _ = gpu_run(ndvm, w)
     idx = np.sort(np.random.default_rng(2).choice(w.B, 64, replace=False))
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(gl[idx], gg[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, sp)
 
 
 def test_kalman_rand8_short(ndvm, oracle_mod, cuda):
     w = W.kalman_rand8(B=40, T=60)
     gl, gg, fl = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(fl, gl)
 
 
@@ -137,8 +137,8 @@ def test_kalman_rand8_full_T_sampled(ndvm, oracle_mod, cuda):
     w = W.kalman_rand8()
     gl, gg, _ = gpu_run(ndvm, w, lanes=1024)
     idx = np.sort(np.random.default_rng(3).choice(1024, 24, replace=False))
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(gl[idx], gg[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, sp)
 
 
 def test_lane_decomposition(ndvm, cuda):
@@ -183,8 +183,8 @@ def test_select_clamps_and_gating(ndvm, oracle_mod, cuda):
     b = np.concatenate([rng.uniform(-2, 2, 60), [0.0, -1e-9, 1.0, -0.5, 0.0]])
     w = W.Workload("select", SELECT_PROG, 0, np.stack([a, b], 1), np.zeros(0), np.zeros(2))
     gl, gg, _ = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
 
 
 def test_empty_batch_and_zero_points(ndvm, cuda):
@@ -217,9 +217,8 @@ def test_logistic_fp32_variant(ndvm, oracle_mod, cuda):
     w = W.logistic(B=300)
     w.params = w.params.astype(np.float32).astype(np.float64)
     gl, gg, fl = gpu_run(ndvm, w, dtype="f32")
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, frontend=w.frontend, nthreads=8,
-                                f32=True)
-    check(gl, gg, ol, og, tol=1e-5)
+    ol, og, sp = oracle_run(oracle_mod, w, f32=True)
+    check(gl, gg, ol, og, sp, tol=1e-5)
     np.testing.assert_array_equal(fl, gl)
 
 
@@ -227,8 +226,8 @@ def test_exp_decay_fp32_variant(ndvm, oracle_mod, cuda):
     w = W.exp_decay(B=64)
     w.params = w.params.astype(np.float32).astype(np.float64)
     gl, gg, _ = gpu_run(ndvm, w, dtype="f32")
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, nthreads=8, f32=True)
-    check(gl, gg, ol, og, tol=1e-5)
+    ol, og, sp = oracle_run(oracle_mod, w, f32=True)
+    check(gl, gg, ol, og, sp, tol=1e-5)
 
 
 ARITH_PROG = """
@@ -268,9 +267,9 @@ def test_zero_adjoints_skip_infinite_factors(ndvm, oracle_mod, cuda):
     b = np.array([800.0, 1e3, 1.0, 30.0, 800.0, 2.0, 40.0])
     w = W.Workload("skip", SKIP_PROG, 0, np.stack([a, b], 1), np.zeros(0), np.zeros(2))
     gl, gg, _ = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
+    ol, og, sp = oracle_run(oracle_mod, w)
     assert np.isfinite(ol).all() and np.isfinite(og).all()  # the pin: every lane stays finite
-    check(gl, gg, ol, og)
+    check(gl, gg, ol, og, sp)
 
 
 def test_async_host_entry_point_overlaps_tapes(ndvm, cuda):
@@ -300,8 +299,8 @@ def test_second_client_bytecode_workloads(ndvm, oracle_mod, cuda, k):
     branch, summed matrix-vector product) over 256 lanes against the oracle."""
     w = W.second_client(B=256)[k]
     gl, gg, fl = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(fl, gl)
 
 
@@ -324,8 +323,8 @@ def test_structural_surface_programs(ndvm, oracle_mod, cuda, name):
     rng = np.random.default_rng(3)
     w = W.Workload(name, STRUCTURAL_PROGRAMS[name], 0, rng.uniform(-1.5, 1.5, (100, 2)), np.zeros(0), np.zeros(2))
     gl, gg, _ = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
 
 
 def test_degenerate_programs(ndvm, oracle_mod, cuda):
@@ -336,8 +335,8 @@ def test_degenerate_programs(ndvm, oracle_mod, cuda):
     w = W.Workload("unused", "(model (params a b c) (* (sin a) (exp c)))", 0,
                    np.random.default_rng(1).normal(size=(37, 3)), np.zeros(0), np.zeros(3))
     gl, gg, _ = gpu_run(ndvm, w)
-    ol, og = oracle_run(oracle_mod, w)
-    check(gl, gg, ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(gl, gg, ol, og, sp)
     np.testing.assert_array_equal(gg[:, 1], 0.0)
     t0 = ndvm.trace_build("(model (params) (* 2.0 (+ 1.5 (obs 0))))")
     p0 = torch.zeros((5, 0), dtype=torch.float64, device="cuda")
@@ -360,8 +359,8 @@ def test_million_lanes_sampled(ndvm, oracle_mod, cuda):
     w = W.Workload("big", base.program, 0, 1.0 + 0.3 * rng.standard_normal((1 << 20, 3)), base.obs, base.truth)
     gl, gg, _ = gpu_run(ndvm, w)
     idx = np.array([0, 1, 12345, 524287, 524288, (1 << 20) - 1])
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(gl[idx], gg[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(gl[idx], gg[idx], ol, og, sp)
 
 
 TWO_REGION_PROG = """
@@ -397,8 +396,8 @@ def test_shared_point_values_match_per_lane_values(ndvm, oracle_mod, cuda, monke
     torch.cuda.synchronize()
     np.testing.assert_array_equal(l1.cpu().numpy(), l2.cpu().numpy())
     np.testing.assert_array_equal(g1.cpu().numpy(), g2.cpu().numpy())
-    ol, og = oracle_run(oracle_mod, w)
-    check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w)
+    check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og, sp)
 
 
 @pytest.mark.parametrize("cfg,B", [(3, 16384), (4, 8192), (6, 256)])
@@ -435,8 +434,8 @@ def test_paired_chains_and_trimmed_fetches_are_exact(ndvm, oracle_mod, cuda, mon
     np.testing.assert_array_equal(l1.cpu().numpy(), l2.cpu().numpy())
     np.testing.assert_array_equal(g1.cpu().numpy(), g2.cpu().numpy())
     idx = np.array([0, 1, B // 2, B - 1])
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(l1.cpu().numpy()[idx], g1.cpu().numpy()[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(l1.cpu().numpy()[idx], g1.cpu().numpy()[idx], ol, og, sp)
 
 
 def _region_workloads():
@@ -478,8 +477,8 @@ def test_point_loads_and_hoisted_seed_are_exact(ndvm, oracle_mod, cuda, monkeypa
     np.testing.assert_array_equal(f1.cpu().numpy(), l1.cpu().numpy())
     B = len(w.params)
     idx = np.array([0, 1, B // 2, B - 1])
-    ol, og = oracle_run(oracle_mod, w, idx)
-    check(l1.cpu().numpy()[idx], g1.cpu().numpy()[idx], ol, og)
+    ol, og, sp = oracle_run(oracle_mod, w, idx)
+    check(l1.cpu().numpy()[idx], g1.cpu().numpy()[idx], ol, og, sp)
 
 
 @pytest.mark.parametrize("name", golden_cases())
@@ -523,5 +522,5 @@ def test_shared_adjoint_slots_stay_apart_where_a_rule_reads_after_writing(ndvm, 
         torch.cuda.synchronize()
         np.testing.assert_array_equal(l1.cpu().numpy(), l2.cpu().numpy())
         np.testing.assert_array_equal(g1.cpu().numpy(), g2.cpu().numpy())
-        ol, og = oracle_run(oracle_mod, w)
-        check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og)
+        ol, og, sp = oracle_run(oracle_mod, w)
+        check(l1.cpu().numpy(), g1.cpu().numpy(), ol, og, sp)

@@ -16,7 +16,7 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import hazard_workloads, matrix_program, rel_check
+from conftest import hazard_workloads, matrix_program, oracle_ref, rel_check
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 CSRC = os.path.join(ROOT, "paper_2607_03574_gb300", "csrc")
@@ -73,8 +73,8 @@ def test_simulated_plans_match_the_oracle_and_each_other(plansim, oracle_mod, k)
     base = simulate(plansim, w, 0)
     if base is None:
         pytest.skip("matrix instructions are not simulated")
-    ol, og = oracle_mod.run(w.program, w.params, w.obs, frontend=w.frontend)
-    ok, rep = rel_check(base[0], base[1], ol, og, 1e-12)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs, frontend=w.frontend)
+    ok, rep = rel_check(base[0], base[1], ol, og, 1e-12, sp)
     assert ok, (w.name, rep)
     value = simulate(plansim, w, 2)
     assert np.array_equal(value[0], base[0]), w.name  # the value-only plan gives the same loss bits
@@ -96,8 +96,8 @@ def test_simulated_matrix_programs(plansim, oracle_mod, k):
     rng = np.random.default_rng(k)
     w = W.Workload(f"matrix_{k}", MATRIX_CASES[k], 0, rng.normal(0.0, 0.5, (6, 4)), np.zeros(0), np.zeros(4))
     base = simulate(plansim, w, 0)
-    ol, og = oracle_mod.run(w.program, w.params, w.obs)
-    ok, rep = rel_check(base[0], base[1], ol, og, 1e-12)
+    ol, og, sp = oracle_ref(oracle_mod, w.program, w.params, w.obs)
+    ok, rep = rel_check(base[0], base[1], ol, og, 1e-12, sp)
     assert ok, (w.program, rep)
     for stream, env in ((1, None), (0, OFF), (1, OFF)):
         other = simulate(plansim, w, stream, env)
