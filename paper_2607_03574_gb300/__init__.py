@@ -69,6 +69,7 @@ def load(build_if_missing: bool = True):
             "ndvm_check_device": (ctypes.c_int, [P]),
             "ndvm_launch_count": (ctypes.c_ulonglong, []),
             "ndvm_measure_fp64_peak": (ctypes.c_int, [ctypes.POINTER(ctypes.c_double), P]),
+            "ndvm_measure_op_cost": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_double), P]),
             "ndvm_last_error": (ctypes.c_char_p, []),
             "ndvm_version": (ctypes.c_char_p, []),
         }
@@ -160,6 +161,17 @@ def measure_fp64_peak(stream=None) -> float:
     return v.value
 
 
+PROBES = ("dfma", "exp", "log", "sin", "cos", "sincos", "tanh", "sqrt", "div", "rcp", "pow", "log_lib", "exp_lib")
+
+
+def measure_op_cost(name: str, iters: int = 2000, stream=None) -> float:
+    """Device time per call (ns, all SMs busy) of one probed function (PROBES)."""
+    v = ctypes.c_double()
+    _check(load().ndvm_measure_op_cost(PROBES.index(name), iters, ctypes.byref(v),
+                                       _stream_ptr(stream) if stream is not None else None))
+    return v.value
+
+
 def _torch():
     import torch
     return torch
@@ -191,12 +203,22 @@ def _dev_ptr(t, name):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _on_stream(stream):
+    """Context in which allocations belong to `stream` (the stream the replay runs on):
+    torch's caching allocator then reuses a freed block only for later work on that
+    stream, never while a kernel queued there may still use it."""
+    torch = _torch()
+    return torch.cuda.stream(stream if stream is not None else torch.cuda.current_stream())
+
+
 def forward(tape: Tape, params, obs, loss=None, stream=None):
-    """Per-lane loss.  params: (B, P) CUDA tensor; obs: 1-d CUDA tensor (same dtype)."""
+    """Per-lane loss.  params: (B, P) CUDA tensor; obs: 1-d CUDA tensor (same dtype).
+    An output this call allocates belongs to `stream` (torch's allocator)."""
     torch = _torch()
     B = params.shape[0]
     if loss is None:
-        loss = torch.empty(B, dtype=params.dtype, device=params.device)
+        with _on_stream(stream):
+            loss = torch.empty(B, dtype=params.dtype, device=params.device)
     _check(load().ndvm_forward(tape.handle, _dtype_code(params), B, _dev_ptr(params, "params"),
                                _dev_ptr(obs, "obs"), 0 if obs is None else obs.numel(), _dev_ptr(loss, "loss"),
                                _stream_ptr(stream)))
@@ -204,17 +226,22 @@ def forward(tape: Tape, params, obs, loss=None, stream=None):
 
 
 class Workspace:
-    """Reusable device workspace for value_and_grad (grown on demand)."""
+    """Reusable device workspace for value_and_grad (grown on demand).  One per
+    (device, stream): it is allocated on the stream its replays run on, so when it
+    grows, the replaced block is not handed to other work while those replays may still
+    read it."""
 
     def __init__(self):
         self.buf = None
 
-    def get(self, nbytes: int, device):
+    def get(self, nbytes: int, device, stream=None):
         torch = _torch()
         if nbytes == 0:
             return None
         if self.buf is None or self.buf.numel() < nbytes or self.buf.device != device:
-            self.buf = torch.empty(nbytes, dtype=torch.uint8, device=device)
+            self.buf = None
+            with _on_stream(stream):
+                self.buf = torch.empty(nbytes, dtype=torch.uint8, device=device)
         return self.buf
 
 
@@ -222,18 +249,21 @@ _default_ws = {}  # (device, stream) -> Workspace: concurrent streams never shar
 
 
 def value_and_grad(tape: Tape, params, obs, loss=None, grad=None, workspace=None, ws_bytes=None, stream=None):
-    """Per-lane loss and gradient.  Returns (loss[B], grad[B, P])."""
+    """Per-lane loss and gradient.  Returns (loss[B], grad[B, P]).  Outputs and the
+    default workspace that this call allocates belong to `stream` (torch's allocator);
+    a caller-given workspace must stay allocated until the replay on `stream` is done."""
     torch = _torch()
     B = params.shape[0]
-    if loss is None:
-        loss = torch.empty(B, dtype=params.dtype, device=params.device)
-    if grad is None:
-        grad = torch.empty_like(params)
+    with _on_stream(stream):
+        if loss is None:
+            loss = torch.empty(B, dtype=params.dtype, device=params.device)
+        if grad is None:
+            grad = torch.empty_like(params)
     dt = _dtype_code(params)
     if workspace is None:
         need = tape.workspace_bytes(B, dt) if ws_bytes is None else ws_bytes
         key = (str(params.device), _stream_ptr(stream).value)
-        workspace = _default_ws.setdefault(key, Workspace()).get(need, params.device)
+        workspace = _default_ws.setdefault(key, Workspace()).get(need, params.device, stream)
     nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     if ws_bytes is not None:
         nbytes = min(nbytes, ws_bytes)
