@@ -588,6 +588,14 @@ ndvm_status ndvm_measure_fp64_peak(double* flops_per_s, void* stream) {
   return NDVM_OK;
 }
 
+ndvm_status ndvm_measure_op_cost(int fn, int iters, double* ns_per_call, void* stream) {
+  if (!ns_per_call) return fail(NDVM_E_INVALID_ARG, "null output");
+  if (fn < 0 || fn >= NDVM_PROBE_COUNT || iters < 1) return fail(NDVM_E_INVALID_ARG, "unknown probe or iters < 1");
+  cudaError_t e = measure_op_cost(fn, iters, ns_per_call, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "function cost probe");
+  return NDVM_OK;
+}
+
 unsigned long long ndvm_launch_count(void) {
   std::lock_guard<std::mutex> lk(g_launch_mu);
   return g_launches;
@@ -608,6 +616,7 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
   if (dtype != NDVM_F64 && dtype != NDVM_F32) return fail(NDVM_E_INVALID_ARG, "bad dtype");
   if (B < 0) return fail(NDVM_E_INVALID_ARG, "B must be >= 0");
   if (B == 0) return NDVM_OK;
+  if (B > (int64_t)1 << 40) return fail(NDVM_E_INVALID_ARG, "B too large");
   const Plan& p = t->grad_plan;
   if (p.n_params > 0 && (!params || !grad)) return fail(NDVM_E_INVALID_ARG, "null params or grad");
   if (!loss) return fail(NDVM_E_INVALID_ARG, "null loss");
@@ -636,6 +645,10 @@ ndvm_status ndvm_value_and_grad_noalloc(const ndvm_tape* tape, ndvm_dtype dtype,
     int64_t fit = (int64_t)(lane_scratch / per_lane);
     if (fit < B) chunk = fit - fit % lanes_per_block;
   }
+  // one launch covers at most kMaxChunk lanes, so its grid stays far below 2^31 blocks
+  if (chunk > kMaxChunk) chunk = kMaxChunk - kMaxChunk % lanes_per_block;
+  if ((chunk + lanes_per_block - 1) / lanes_per_block > 0x7fffffff)
+    return fail(NDVM_E_INVALID_ARG, "too many lanes for one launch");
   DevCache* dc = nullptr;
   {
     int dev = 0;

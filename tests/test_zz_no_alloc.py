@@ -13,7 +13,6 @@ import numpy as np
 import pytest
 
 import workloads as W
-from conftest import rel_check
 
 pytestmark = pytest.mark.gpu
 
@@ -28,26 +27,41 @@ def _noalloc(nd, tape, p, o, loss, grad):
         ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
 
 
-@pytest.mark.parametrize("make", [lambda: W.logistic(B=3000), lambda: W.random_exprs(2, B=700, n_points=256)[1]],
+SCRATCH_BYTES = 32 << 20
+
+
+@pytest.mark.parametrize("make", [lambda: W.logistic(B=3000), lambda: W.random_exprs(1, B=3000, n_points=256)[0]],
                          ids=["workspace-tape", "data-axis-tape"])
 def test_noalloc_matches_regular_entry_point_twice(ndvm, cuda, make):
+    """Two calls in a row with different inputs and lane counts (3000 lanes; then the last
+    1537 lanes with every parameter scaled by 1.05 and the observations by 0.9), each
+    equal bit for bit to ndvm_value_and_grad on the same inputs: the second call must
+    not read what the first left in the shared scratch.  The logistic tape keeps 4,099
+    values per lane, so its 3000 lanes (98 MB) run in more than one launch over the
+    32 MiB scratch; the random-expression tape keeps its per-point values shared by all
+    lanes (computed from the observations) at the start of the scratch."""
     import torch
     w = make()
     tape = ndvm.trace_build(w.program, w.frontend)
-    p = torch.tensor(w.params, dtype=torch.float64, device="cuda")
-    o = torch.tensor(w.obs, dtype=torch.float64, device="cuda")
-    ref_loss, ref_grad = ndvm.value_and_grad(tape, p, o)  # also makes the tape resident
-    torch.cuda.synchronize()
-    rl, rg = ref_loss.cpu().numpy(), ref_grad.cpu().numpy()
-    loss, grad = torch.empty_like(ref_loss), torch.empty_like(ref_grad)  # outputs come from the caller
-    for _ in range(2):
-        loss.fill_(float("nan"))
-        grad.fill_(float("nan"))
+    assert tape.cost()["save_elems"] > 0 or tape.cost()["work_shared"] > 0
+    for params, obs in ((w.params, w.obs), (w.params[-1537:] * 1.05, w.obs * 0.9)):
+        B = len(params)
+        p = torch.tensor(params, dtype=torch.float64, device="cuda")
+        o = torch.tensor(obs, dtype=torch.float64, device="cuda")
+        ref_loss, ref_grad = ndvm.value_and_grad(tape, p, o)  # also makes the tape resident
+        torch.cuda.synchronize()
+        loss, grad = torch.full_like(ref_loss, float("nan")), torch.full_like(ref_grad, float("nan"))
+        n0 = ndvm.launch_count()
         st = _noalloc(ndvm, tape, p, o, loss, grad)
         assert st == 0, ndvm.load().ndvm_last_error()
+        launches = ndvm.launch_count() - n0
         torch.cuda.synchronize()
-        ok, rep = rel_check(loss.cpu().numpy(), grad.cpu().numpy(), rl, rg, 1e-12)
-        assert ok, rep
+        ndvm.check_device(tape)
+        np.testing.assert_array_equal(loss.cpu().numpy(), ref_loss.cpu().numpy())
+        np.testing.assert_array_equal(grad.cpu().numpy(), ref_grad.cpu().numpy())
+        saves = tape.cost()["save_elems"]
+        if saves and B == 3000:
+            assert saves * 8 * B > SCRATCH_BYTES and launches > 1, (saves, B, launches)
 
 
 def test_noalloc_refuses_instead_of_allocating(ndvm, cuda):
