@@ -201,6 +201,25 @@ ndvm_status ndvm_tape_shared_work(const ndvm_tape* tape, double* work_per_call);
  */
 ndvm_status ndvm_measure_fp64_peak(double* flops_per_s, void* stream);
 
+/* Functions that ndvm_measure_op_cost times (the replay's own exp and log, CUDA's
+ * other functions, and DFMA as the unit). */
+enum {
+  NDVM_PROBE_DFMA = 0, NDVM_PROBE_EXP = 1, NDVM_PROBE_LOG = 2, NDVM_PROBE_SIN = 3, NDVM_PROBE_COS = 4,
+  NDVM_PROBE_SINCOS = 5, NDVM_PROBE_TANH = 6, NDVM_PROBE_SQRT = 7, NDVM_PROBE_DIV = 8, NDVM_PROBE_RCP = 9,
+  NDVM_PROBE_POW = 10, NDVM_PROBE_LOGLIB = 11, NDVM_PROBE_EXPLIB = 12, NDVM_PROBE_COUNT = 13
+};
+
+/*
+ * ndvm_measure_op_cost -- device time per call (ns, every SM busy with four
+ * independent chains per thread, 1024 threads per SM) of the function `fn`
+ * (NDVM_PROBE_*), each call followed by one FP64 add.  Dividing by the DFMA probe's
+ * time gives the function's throughput cost in DFMA-equivalents; an ncu capture of
+ * the probe launch gives its FP64-pipe instructions per call (calls = 4 x iters x
+ * threads).  The paper has no counterpart: it measures the denominators of the
+ * roofline.  Synchronous; NDVM_E_INVALID_ARG for an unknown fn or iters < 1.
+ */
+ndvm_status ndvm_measure_op_cost(int fn, int iters, double* ns_per_call, void* stream);
+
 /* ndvm_launch_count -- replay kernels launched by this process so far. */
 unsigned long long ndvm_launch_count(void);
 

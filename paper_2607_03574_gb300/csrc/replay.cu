@@ -27,6 +27,7 @@
 #include <map>
 #include <mutex>
 
+#include "ndvm.h"
 #include "plan.h"
 #include "replay.h"
 #include "fmath.cuh"
@@ -916,6 +917,91 @@ cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s) {
   cudaEventDestroy(e1);
   cudaFree(out);
   if (e == cudaSuccess) *flops_per_s = 2.0 * 8.0 * iters * (double)blocks * threads / (best * 1e-3);
+  return e;
+}
+}  // namespace ndvm
+
+// ---------------------------------------------------------------------------
+// Per-function cost probe: the throughput of one library function (or of the
+// replay's own exp and log) relative to DFMA, for the roofline's cost table.  Every
+// thread runs four independent chains x <- f(x) + c (c keeps x in the function's
+// ordinary domain); one FP64 add per call is part of the chain and is counted in the
+// measured time.  Launch shape and iteration count match the FP64 peak probe's
+// per-thread work, so an ncu capture of a probe launch gives the function's FP64-pipe
+// instructions per call (calls = blocks x threads x iters x 4).
+namespace ndvm {
+namespace {
+template <int FN>
+__device__ __forceinline__ double probe_f(double x) {
+  switch (FN) {
+    case NDVM_PROBE_DFMA: return fma(x, 0.999999999, 1e-9);
+    case NDVM_PROBE_EXP: return fast_exp(-x) + 0.25;
+    case NDVM_PROBE_LOG: return fast_log(x) + 2.0;
+    case NDVM_PROBE_SIN: return sin(x) + 1.0;
+    case NDVM_PROBE_COS: return cos(x) + 1.0;
+    case NDVM_PROBE_SINCOS: { double s, c; sincos(x, &s, &c); return s + c; }
+    case NDVM_PROBE_TANH: return tanh(x) + 0.5;
+    case NDVM_PROBE_SQRT: return sqrt(x) + 1.0;
+    case NDVM_PROBE_DIV: return 3.0 / (x + 1.0);
+    case NDVM_PROBE_RCP: return 1.0 / x + 0.5;
+    case NDVM_PROBE_POW: return pow(x, 0.75) + 1.0;
+    case NDVM_PROBE_LOGLIB: return log(x) + 2.0;
+    case NDVM_PROBE_EXPLIB: return exp(-x) + 0.25;
+    default: return x;
+  }
+}
+template <int FN>
+__global__ void __launch_bounds__(256) k_op_probe(double* out, int iters) {
+  double a[4];
+#pragma unroll
+  for (int k = 0; k < 4; k++) a[k] = 1.0 + 0.125 * k + 1e-7 * threadIdx.x;
+  for (int i = 0; i < iters; i++) {
+#pragma unroll
+    for (int k = 0; k < 4; k++) a[k] = probe_f<FN>(a[k]);
+  }
+  out[(size_t)blockIdx.x * blockDim.x + threadIdx.x] = a[0] + a[1] + a[2] + a[3];
+}
+template <int FN>
+void launch_probe(double* out, int blocks, int iters, cudaStream_t s) {
+  k_op_probe<FN><<<blocks, 256, 0, s>>>(out, iters);
+}
+using ProbeFn = void (*)(double*, int, int, cudaStream_t);
+constexpr ProbeFn kProbes[NDVM_PROBE_COUNT] = {
+    launch_probe<0>, launch_probe<1>, launch_probe<2>, launch_probe<3>, launch_probe<4>,
+    launch_probe<5>, launch_probe<6>, launch_probe<7>, launch_probe<8>, launch_probe<9>,
+    launch_probe<10>, launch_probe<11>, launch_probe<12>};
+}  // namespace
+
+cudaError_t measure_op_cost(int fn, int iters, double* ns_per_call, cudaStream_t s) {
+  if (fn < 0 || fn >= NDVM_PROBE_COUNT || iters < 1) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  const int blocks = sms * 4, threads = 256;
+  double* out = nullptr;
+  if ((e = cudaMalloc(&out, sizeof(double) * blocks * threads)) != cudaSuccess) return e;
+  cudaEvent_t e0, e1;
+  cudaEventCreate(&e0);
+  cudaEventCreate(&e1);
+  kProbes[fn](out, blocks, 16, s);  // warm-up
+  float best = 1e30f;
+  for (int rep = 0; rep < 3; rep++) {
+    cudaEventRecord(e0, s);
+    kProbes[fn](out, blocks, iters, s);
+    cudaEventRecord(e1, s);
+    e = cudaEventSynchronize(e1);
+    if (e != cudaSuccess) break;
+    float ms = 0;
+    cudaEventElapsedTime(&ms, e0, e1);
+    if (ms < best) best = ms;
+  }
+  if (e == cudaSuccess) e = cudaGetLastError();
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  cudaFree(out);
+  // device time per call, all SMs busy: total time / calls
+  if (e == cudaSuccess) *ns_per_call = best * 1e6 / (4.0 * iters * (double)blocks * threads);
   return e;
 }
 }  // namespace ndvm

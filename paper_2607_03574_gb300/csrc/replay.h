@@ -44,4 +44,7 @@ cudaError_t noalloc_scratch(void** ptr);
 // Measured FP64 fused multiply-add throughput of the current device (flop/s, 2 per FMA).
 cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s);
 
+// Device time per call of one probed function (NDVM_PROBE_*), every SM busy.
+cudaError_t measure_op_cost(int fn, int iters, double* ns_per_call, cudaStream_t s);
+
 }  // namespace ndvm
