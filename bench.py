@@ -4,9 +4,17 @@ One step = the whole hot path over one batch: 200 seeded random-expression progr
 (grammar + - * / exp log|x| sin pow-int, depth <= 6, 1-8 constants), each replayed
 forward and in reverse over B = 4096 parameter lanes and 256 data points (MSE loss)
 -- 819,200 lane value+grad evaluations.  Inputs are resident in HBM before the timed
-region; L2 is flushed between timed steps.  Prints one JSON line.
+region; L2 is flushed between timed steps.  Prints one JSON line: the headline
+configuration's numbers, and under "configs" the same measurement of every other
+configuration (exp-decay, logistic f64 and f32, the two Kalman filters, the 64-state
+population), each with a bounded CPU-oracle baseline.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+                    [--config C] [--dtype f32] [--only]
+
+Under N processes (one per GPU) the population has N x 4096 lanes per program; rank r
+replays lanes [4096 r, 4096 (r + 1)) of every program (weak scaling) and rank 0 gathers
+the slices of loss and gradient on the host after the timed region.
 
 --impl reference times the oracle (the plain CPU reference evaluator) on the host
 cores instead, on a bounded sample of the same workload.
@@ -57,7 +65,7 @@ def kernel_sources_digest():
     return h.hexdigest()
 
 
-def recorded_traffic(args, n_programs):
+def recorded_traffic(cfg: int, dtype: str, lanes: int, n_programs: int):
     """DRAM bytes (read + write) per replay launch from the committed ncu summary of this
     workload, if the library's sources are the ones it was taken from; else None."""
     try:
@@ -65,12 +73,11 @@ def recorded_traffic(args, n_programs):
             rec = json.load(f)
     except (OSError, ValueError):
         return None
-    if rec.get("sources_sha256") != kernel_sources_digest() or args.dtype != "f64":
+    if rec.get("sources_sha256") != kernel_sources_digest() or dtype != "f64":
         return None
-    key = str(args.config)
-    if args.lanes or (args.config == 2 and n_programs != N_PROGRAMS):
+    if lanes or (cfg == 2 and n_programs != N_PROGRAMS):
         return None
-    ent = rec.get("per_launch", {}).get(key)
+    ent = rec.get("per_launch", {}).get(str(cfg))
     return None if ent is None else float(ent["dram_bytes"])
 
 
@@ -79,11 +86,6 @@ def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return rank, world, local
-
-
-def rank_seed(rank: int) -> int:
-    """Each rank replays its own seeded population (weak scaling: per-GPU work fixed)."""
-    return SEED + 7919 * rank
 
 
 def max_over_ranks(ms: float, device=None) -> float:
@@ -151,21 +153,40 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def workload_for(args, seed):
-    """(list of Workloads, description) of the configuration being measured."""
-    if args.config == 2:
-        B = args.lanes or B_LANES
-        progs = W.random_exprs(n_programs=args.programs, B=B, n_points=N_POINTS, seed=seed)
-        desc = (f"random-expression programs: {len(progs)} programs x {B} lanes x {N_POINTS} points, "
-                f"MSE, {args.dtype} value+grad")
-        return progs, desc
-    w = W.config(args.config, seed=seed, **({"B": args.lanes} if args.lanes else {}))
-    desc = {1: f"exp-decay y = a exp(-b t) + c: {w.B} lanes x 50 points, MSE",
-            3: f"logistic Euler (stack bytecode): {w.B} lanes x 1000 steps, 100 obs, MSE",
-            4: f"4-state constant-velocity Kalman NLL: {w.B} lanes x 200 steps",
-            5: f"8-state random stable Kalman NLL: {w.B} lanes x 1000 steps",
-            6: f"64-state Kalman NLL population, 8-d observations: {w.B} lanes x 50 steps"}[args.config]
-    return [w], f"{desc}, {args.dtype} value+grad"
+DEFAULT_LANES = {1: 64, 2: B_LANES, 3: 16384, 4: 8192, 5: 65536, 6: 1024}
+DESCRIPTIONS = {1: "exp-decay y = a exp(-b t) + c: {B} lanes x 50 points, MSE",
+                3: "logistic Euler (stack bytecode): {B} lanes x 1000 steps, 100 obs, MSE",
+                4: "4-state constant-velocity Kalman NLL: {B} lanes x 200 steps",
+                5: "8-state random stable Kalman NLL: {B} lanes x 1000 steps",
+                6: "64-state Kalman NLL population, 8-d observations: {B} lanes x 50 steps"}
+
+
+def population(args, cfg: int, world: int = 1, rank: int = 0, lanes_per_rank: int = 0):
+    """(this rank's Workloads, description, lanes per program in the whole population).
+
+    One seeded population of world x lanes_per_rank lanes per program (the generator's
+    population at that size); this rank's Workloads hold its slice of the lanes
+    (shard.lane_slice), the same programs and observations on every rank."""
+    from dataclasses import replace
+
+    from paper_2607_03574_gb300.shard import lane_slice
+    B_rank = lanes_per_rank or DEFAULT_LANES[cfg]
+    B_total = B_rank * world
+    if cfg == 2:
+        progs = W.random_exprs(n_programs=args.programs, B=B_total, n_points=N_POINTS, seed=SEED)
+        desc = (f"random-expression programs: {len(progs)} programs x {B_total} lanes x {N_POINTS} points, MSE")
+    else:
+        progs = [W.config(cfg, B=B_total, seed=SEED)]
+        desc = DESCRIPTIONS[cfg].format(B=B_total)
+    lo, hi = lane_slice(B_total, world, rank)
+    local = [replace(w, params=w.params[lo:hi]) for w in progs]
+    return local, desc, B_total
+
+
+def workload_for(args, seed=SEED):
+    """(list of Workloads, description) of the configuration being measured, one process."""
+    progs, desc, _ = population(args, args.config, 1, 0, args.lanes)
+    return progs, f"{desc}, {args.dtype} value+grad"
 
 
 def cpu_sample_lanes(args, progs):
@@ -216,6 +237,20 @@ def cpu_baseline(args, progs):
                                       f"evals ({dt1:.1f} s)"}}
 
 
+def bounded_cpu_baseline(progs, f32: bool, seconds: float = 2.0):
+    """The oracle on every host core over a sample sized to take about `seconds`: a short
+    probe on a few lanes gives the rate, which sizes the timed sample (a prefix of the
+    population's lanes, the same for every program)."""
+    cores = os.cpu_count() or 1
+    probe = max(1, min(progs[0].B, cores))
+    n, dt = oracle_sample_time(progs, probe, cores, f32, tile=False)
+    lanes = int(min(progs[0].B, max(probe, (n / dt) * seconds / len(progs))))
+    n, dt = oracle_sample_time(progs, lanes, cores, f32, tile=False)
+    return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"the first {lanes} of {progs[0].B} lanes of each of the {len(progs)} program(s): "
+                      f"{n} lane evals in {dt:.1f} s"}
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -246,54 +281,26 @@ def run_reference(args):
     return 0
 
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
-    ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
-    ap.add_argument("--programs", type=int, default=N_PROGRAMS, help="programs per step (smaller for profiling)")
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6],
-                    help="workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other configurations; "
-                         "6 a 64-state Kalman population (block-cooperative lanes)")
-    ap.add_argument("--dtype", default="f64", choices=["f64", "f32"])
-    ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
-    ap.add_argument("--cpu-lanes", type=int, default=0,
-                    help="oracle lanes per program for cpu_baseline (default: 2048 for the random programs, "
-                         "every lane otherwise)")
-    ap.add_argument("--lanes", type=int, default=0, help="lanes per program instead of the configuration's "
-                                                         "(smaller cases for profiling)")
-    ap.add_argument("--streams", type=int, default=16, help="CUDA streams the programs are spread over")
-    ap.add_argument("--no-graph", dest="graph", action="store_false",
-                    help="launch every step from the host instead of replaying a captured CUDA graph")
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    args = ap.parse_args()
-    if args.warmup < 3:
-        ap.error("--warmup must be >= 3")
-    if args.impl == "reference":
-        return run_reference(args)
+NOMINAL_FP64_TFLOPS = 1.25  # GB300 nominal FP64 rate (context; the roofline uses the measured rate)
 
+
+def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peak_flops, want_gather):
+    """Time one configuration: W warm-up steps, then K timed steps of a captured CUDA
+    graph of one whole step (every program of this rank's slice), L2 flushed before
+    each; then the same work end to end through the host-buffer entry point.  Returns
+    the measurement and, on rank 0 when want_gather, the population gathered from every
+    rank's slice."""
     import torch
-    import paper_2607_03574_gb300 as nd
 
-    rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    nd.load()
-
-    # ---- workload: programs traced once on the host; inputs resident in HBM
-    progs, workload = workload_for(args, rank_seed(rank))
-    tdt = torch.float32 if args.dtype == "f32" else torch.float64
-    npdt = np.float32 if args.dtype == "f32" else np.float64
+    tdt = torch.float32 if dtype == "f32" else torch.float64
+    npdt = np.float32 if dtype == "f32" else np.float64
+    progs = local_progs
     t0 = time.perf_counter()
     tapes = [nd.trace_build(w.program, w.frontend) for w in progs]
     trace_s = time.perf_counter() - t0
     params = [torch.tensor(w.params, dtype=tdt, device=dev) for w in progs]
     obs = [torch.tensor(w.obs, dtype=tdt, device=dev) for w in progs]
-    loss = [torch.empty(w.B, dtype=torch.float64, device=dev) for w in progs]
+    loss = [torch.empty(w.B, dtype=tdt, device=dev) for w in progs]
     grad = [torch.empty_like(p) for p in params]
     flush = torch.empty(256 * 1024 * 1024, dtype=torch.uint8, device=dev)  # > 129 MB L2
     stream = torch.cuda.current_stream(dev)
@@ -306,11 +313,12 @@ def main():
         alg_bytes += (2 * c["save_elems"] + 2 * w.P + 1) * esz * w.B + esz * w.obs.size
 
     # independent programs run on several streams so their kernels co-reside on the SMs
-    side = [torch.cuda.Stream(dev) for _ in range(args.streams)]
+    n_streams = min(args.streams, len(tapes))
+    side = [torch.cuda.Stream(dev) for _ in range(n_streams)]
 
     def step():
         cur = torch.cuda.current_stream(dev)  # the capture stream while a graph is captured
-        if args.streams <= 1:
+        if n_streams <= 1:
             for k in range(len(tapes)):
                 nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=cur)
             return
@@ -319,7 +327,7 @@ def main():
         done = []
         for j, s in enumerate(side):
             s.wait_event(start)
-            for k in range(j, len(tapes), args.streams):
+            for k in range(j, len(tapes), n_streams):
                 nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=s)
             e = torch.cuda.Event()
             e.record(s)
@@ -344,17 +352,13 @@ def main():
         torch.cuda.synchronize()
     run_step = graph.replay if graph is not None else step
 
-    torch.cuda.synchronize()
-    peak_flops = nd.measure_fp64_peak()
-
-    clocks = ClockSampler(local)
+    clocks = ClockSampler(dev.index)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     clocks.start()
     time.sleep(0.3)
     l0 = nd.launch_count()
-    step_ms = []
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     wall0 = time.perf_counter()
     for i in range(args.steps):
@@ -364,19 +368,36 @@ def main():
         ev[i][1].record(stream)
     torch.cuda.synchronize()
     wall = time.perf_counter() - wall0
+    if world > 1:
+        torch.distributed.barrier()
     launches = nd.launch_count() - l0 + per_step_launches * args.steps
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    ms = max_over_ranks(float(np.mean(step_ms)), dev)
+    ms = max_over_ranks(float(statistics.median(step_ms)), dev)
+    ms_mean = max_over_ranks(float(np.mean(step_ms)), dev)
     clk = clocks.stop()
     lanes_per_step = sum(w.B for w in progs) * world
     value = lanes_per_step / (ms * 1e-3)
+    for t in tapes:
+        nd.check_device(t)
+
+    gathered = None
+    if want_gather and world > 1:
+        from paper_2607_03574_gb300.shard import gather_lanes
+        ok = True
+        for k in range(len(tapes)):
+            ll, gg = loss[k].double().cpu().numpy(), grad[k].double().cpu().numpy()
+            gl = gather_lanes(ll, B_total, world, rank, group=args.host_group)
+            gg_all = gather_lanes(gg, B_total, world, rank, group=args.host_group)
+            if rank == 0:
+                ok &= gl.shape == (B_total,) and gg_all.shape == (B_total, gg.shape[1])
+                ok &= bool(np.array_equal(gl[: len(ll)], ll)) and bool(np.array_equal(gg_all[: len(gg)], gg))
+        gathered = {"lanes_per_program": B_total, "programs": len(tapes), "rank0_slice_intact": bool(ok)}
 
     # ---- end to end through the host-buffer entry point (pinned host memory)
     hp = [torch.tensor(w.params, dtype=tdt).pin_memory().numpy() for w in progs]
     ho = [torch.tensor(w.obs, dtype=tdt).pin_memory().numpy() for w in progs]
     h2d = sum(a.nbytes for a in hp) + sum(a.nbytes for a in ho)
-    d2h = sum(w.B * np.dtype(npdt).itemsize * (1 + w.P) for w in progs)
-
+    d2h = sum(w.B * esz * (1 + w.P) for w in progs)
     hl = [torch.empty(w.B, dtype=tdt).pin_memory().numpy() for w in progs]
     hg = [torch.empty((w.B, w.P), dtype=tdt).pin_memory().numpy() for w in progs]
 
@@ -393,7 +414,7 @@ def main():
         t1 = time.perf_counter()
         e2e_step()
         e2e_times.append(time.perf_counter() - t1)
-    e2e_value = lanes_per_step / float(np.mean(e2e_times)) if world == 1 else None
+    e2e_value = lanes_per_step / float(np.median(e2e_times)) if world == 1 else None
 
     # ---- roofline of the replay kernel: the slower of the FP64 work at the measured
     # FP64 rate and the algorithmic bytes at the measured HBM bandwidth, against the
@@ -404,8 +425,9 @@ def main():
     roofline = {
         "bound": "alu", "achieved": achieved / 1e12, "peak": peak_flops / 1e12, "unit": "TFLOP/s",
         "frac": max(t_fp64, t_hbm) / (ms * 1e-3),
-        "traffic": recorded_traffic(args, len(progs)),
+        "traffic": recorded_traffic(cfg, dtype, args.lanes, len(tapes)),
         "peak_source": "FP64 FMA rate measured in this process (8 chains/thread, 4x256 threads/SM)",
+        "nominal_peak": NOMINAL_FP64_TFLOPS, "frac_of_nominal": achieved / (NOMINAL_FP64_TFLOPS * 1e12),
         "work_dfma_per_step": work,
         "hbm_term": {"algorithmic_bytes_per_step": alg_bytes, "peak_gbs": hbm_gbs, "peak_source": hbm_src,
                      "ms_at_peak": 1e3 * t_hbm, "fp64_ms_at_peak": 1e3 * t_fp64,
@@ -413,27 +435,132 @@ def main():
     }
     if t_hbm > t_fp64:
         roofline.update({"bound": "hbm", "achieved": alg_bytes / (ms * 1e-3) / 1e9, "peak": hbm_gbs, "unit": "GB/s"})
+    if dtype == "f32":
+        # the cost table counts FP64 work; the fp32 variant runs on the FP32 pipe, whose
+        # rate is far higher, so no FP64 fraction describes it
+        roofline.update({"frac": None, "frac_of_nominal": None,
+                         "note": "fp32 variant: the FP64 cost model does not apply; frac not reported"})
+    out = {"value": value, "unit": UNIT, "ms_per_step": ms, "ms_per_step_mean": ms_mean,
+           "step_ms": step_ms if world == 1 else None, "lanes_per_step": lanes_per_step,
+           "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+           "gpu_launches": launches, "graph": graph is not None, "roofline": roofline, "clocks": clk,
+           "wall_s_timed": wall, "trace_build_s": trace_s}
+    if gathered is not None:
+        out["gathered_on_rank0"] = gathered
+    del tapes, params, obs, loss, grad, flush, graph
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return out
 
+
+EXTRA = [(1, "f64"), (3, "f64"), (3, "f32"), (4, "f64"), (5, "f64"), (6, "f64")]
+PROBE_ITERS = 2000
+
+
+def probe_costs():
+    """Device time per call of every probed function, all SMs busy, and its ratio to a
+    DFMA's (each probed call carries one FP64 add, which the ratio leaves in: subtract 1
+    for the function alone).  With an ncu capture of the same launches (one per function,
+    after one warm-up launch each), FP64-pipe instructions per call = the launch's
+    smsp__inst_executed_pipe_fp64.sum x 32 / calls."""
+    import torch
+    import paper_2607_03574_gb300 as nd
+    nd.load()
+    torch.cuda.set_device(0)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    calls = 4 * PROBE_ITERS * sms * 4 * 256
+    ns = {name: nd.measure_op_cost(name, PROBE_ITERS) for name in nd.PROBES}
+    out = {"unit": "ns per call (device time, all SMs busy) and DFMA-equivalents (incl. one FP64 add)",
+           "iters": PROBE_ITERS, "calls_per_launch": calls,
+           "ns_per_call": ns, "dfma_equivalents": {k: v / ns["dfma"] for k, v in ns.items()}}
+    print(json.dumps(out), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ndvm", choices=["ndvm", "reference"])
+    ap.add_argument("--programs", type=int, default=N_PROGRAMS, help="programs per step (smaller for profiling)")
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6],
+                    help="headline workload: 2 (default) random-expression programs; 1, 3, 4, 5 the other "
+                         "configurations; 6 a 64-state Kalman population (block-cooperative lanes)")
+    ap.add_argument("--dtype", default="f64", choices=["f64", "f32"])
+    ap.add_argument("--only", action="store_true",
+                    help="measure the headline configuration only (no per-configuration table)")
+    ap.add_argument("--ref-lanes", type=int, default=256, help="oracle lanes per program per reference step")
+    ap.add_argument("--cpu-lanes", type=int, default=0,
+                    help="oracle lanes per program for cpu_baseline (default: 2048 for the random programs, "
+                         "every lane otherwise)")
+    ap.add_argument("--lanes", type=int, default=0, help="lanes per program and rank instead of the "
+                                                         "configuration's (smaller cases for profiling)")
+    ap.add_argument("--streams", type=int, default=16, help="CUDA streams the programs are spread over")
+    ap.add_argument("--no-graph", dest="graph", action="store_false",
+                    help="launch every step from the host instead of replaying a captured CUDA graph")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--probe-costs", action="store_true",
+                    help="print each library function's measured throughput cost in DFMA-equivalents and exit")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    if args.probe_costs:
+        return probe_costs()
+
+    import torch
+    import paper_2607_03574_gb300 as nd
+
+    rank, world, local = dist_env()
+    args.host_group = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+        args.host_group = dist.new_group(backend="gloo")  # host-side gather of the lane slices
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    nd.load()
+    peak_flops = nd.measure_fp64_peak()
+
+    progs, desc, B_total = population(args, args.config, world, rank, args.lanes)
+    head = measure(nd, dev, progs, B_total, args.config, args.dtype, args, world, rank, peak_flops, True)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, progs)
 
+    configs = {}
+    if not args.only and not args.lanes:
+        for cfg, dt in EXTRA:
+            if (cfg, dt) == (args.config, args.dtype):
+                continue
+            p2, d2, bt2 = population(args, cfg, world, rank, 0)
+            m = measure(nd, dev, p2, bt2, cfg, dt, args, world, rank, peak_flops, False)
+            m["workload"] = f"{d2}, {dt} value+grad"
+            if rank == 0 and not args.no_cpu_baseline:
+                m["cpu_baseline"] = bounded_cpu_baseline(p2, dt == "f32")
+            configs[f"{cfg}" if dt == "f64" else f"{cfg}_{dt}"] = m
+
     if rank == 0:
+        cfg_key = {"workload": f"{desc}, {args.dtype} value+grad", "programs": len(progs),
+                   "lanes_per_program": B_total, "lanes_per_rank": progs[0].B, "points": N_POINTS, "seed": SEED,
+                   "l2": "flushed (256 MB write) before every timed step",
+                   "parallelism": f"one population, lanes sliced across ranks (dp{world}); host gather on rank 0",
+                   "streams": args.streams, "step_time": "median of the timed steps (max over ranks)"}
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": args.dtype, "data": "synthetic",
-            "config": {"workload": workload, "programs": len(progs), "lanes_per_program": progs[0].B,
-                       "points": N_POINTS, "seed": SEED, "l2": "flushed (256 MB write) before every timed step",
-                       "parallelism": f"lanes sharded, dp{world}", "streams": args.streams},
-            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-            "gpu_launches": launches, "graph": graph is not None,
-            "roofline": roofline,
-            "cpu_baseline": cpu,
-            "clocks": clk,
-            "wall_s_timed": wall,
-            "trace_build_s": trace_s,
+            "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": head["ms_per_step"], "ms_per_step_mean": head["ms_per_step_mean"],
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": args.dtype,
+            "data": "synthetic", "config": cfg_key, "e2e": head["e2e"], "gpu_launches": head["gpu_launches"],
+            "graph": head["graph"], "roofline": head["roofline"], "cpu_baseline": cpu, "clocks": head["clocks"],
+            "wall_s_timed": head["wall_s_timed"], "trace_build_s": head["trace_build_s"],
+            "step_ms": head["step_ms"],
         }
+        if "gathered_on_rank0" in head:
+            line["gathered_on_rank0"] = head["gathered_on_rank0"]
+        if configs:
+            line["configs"] = configs
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
