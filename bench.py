@@ -281,10 +281,24 @@ def run_reference(args):
     return 0
 
 
-NOMINAL_FP64_TFLOPS = 1.25  # GB300 nominal FP64 rate (context; the roofline uses the measured rate)
+NOMINAL_FP64_TFLOPS = 1.25  # GB300 nominal FP64 rate (context)
+FP64_DFMA_PER_CLK_PER_SM = 2.0  # the FP64 pipe: 16 active cycles per 32-lane warp instruction (ncu)
 
 
-def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peak_flops, want_gather):
+def fp64_pipe_peak(sms: int) -> tuple[float, str]:
+    """Peak FP64 rate from unit counts and clocks (flop/s, 2 per DFMA): 2 DFMA per clock
+    per SM x SMs x the maximum SM clock (MEASURED_PEAKS.json sm_max_mhz, else 2070 MHz)."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            mhz, src = float(json.load(f)["sm_max_mhz"]), "MEASURED_PEAKS.json sm_max_mhz"
+    except (OSError, KeyError, ValueError):
+        mhz, src = 2070.0, "GB300 maximum SM clock 2070 MHz"
+    return (2.0 * FP64_DFMA_PER_CLK_PER_SM * sms * mhz * 1e6,
+            f"FP64 pipe peak from unit counts: {FP64_DFMA_PER_CLK_PER_SM:g} DFMA/clk/SM x {sms} SMs x {mhz:g} MHz "
+            f"({src}); ncu's FP64-pipe utilisation is relative to the same rate")
+
+
+def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks, want_gather):
     """Time one configuration: W warm-up steps, then K timed steps of a captured CUDA
     graph of one whole step (every program of this rank's slice), L2 flushed before
     each; then the same work end to end through the host-buffer entry point.  Returns
@@ -416,17 +430,21 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peak_f
         e2e_times.append(time.perf_counter() - t1)
     e2e_value = lanes_per_step / float(np.median(e2e_times)) if world == 1 else None
 
-    # ---- roofline of the replay kernel: the slower of the FP64 work at the measured
-    # FP64 rate and the algorithmic bytes at the measured HBM bandwidth, against the
+    # ---- roofline of the replay kernel: the slower of the FP64 work at the FP64 pipe's
+    # peak rate and the algorithmic bytes at the measured HBM bandwidth, against the
     # step's kernel time (all launches of a step; they overlap on the streams)
+    pipe_peak, pipe_src, probe_peak = peaks
     achieved = 2.0 * work / (ms * 1e-3)  # flop/s (2 per DFMA-equivalent)
     hbm_gbs, hbm_src = measured_hbm_gbs()
-    t_fp64, t_hbm = 2.0 * work / peak_flops, alg_bytes / (hbm_gbs * 1e9)
+    t_fp64, t_hbm = 2.0 * work / pipe_peak, alg_bytes / (hbm_gbs * 1e9)
     roofline = {
-        "bound": "alu", "achieved": achieved / 1e12, "peak": peak_flops / 1e12, "unit": "TFLOP/s",
+        "bound": "alu", "achieved": achieved / 1e12, "peak": pipe_peak / 1e12, "unit": "TFLOP/s",
         "frac": max(t_fp64, t_hbm) / (ms * 1e-3),
         "traffic": recorded_traffic(cfg, dtype, args.lanes, len(tapes)),
-        "peak_source": "FP64 FMA rate measured in this process (8 chains/thread, 4x256 threads/SM)",
+        "peak_source": pipe_src,
+        "peak_probe": probe_peak / 1e12, "frac_of_probe": achieved / probe_peak,
+        "probe_source": "DFMA stream measured in this process (8 chains/thread, 4x256 threads/SM): "
+                        "ncu shows the FP64 pipe 84 % active there, one warp instruction per 19 cycles per SM",
         "nominal_peak": NOMINAL_FP64_TFLOPS, "frac_of_nominal": achieved / (NOMINAL_FP64_TFLOPS * 1e12),
         "work_dfma_per_step": work,
         "hbm_term": {"algorithmic_bytes_per_step": alg_bytes, "peak_gbs": hbm_gbs, "peak_source": hbm_src,
@@ -438,7 +456,7 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peak_f
     if dtype == "f32":
         # the cost table counts FP64 work; the fp32 variant runs on the FP32 pipe, whose
         # rate is far higher, so no FP64 fraction describes it
-        roofline.update({"frac": None, "frac_of_nominal": None,
+        roofline.update({"frac": None, "frac_of_nominal": None, "frac_of_probe": None,
                          "note": "fp32 variant: the FP64 cost model does not apply; frac not reported"})
     out = {"value": value, "unit": UNIT, "ms_per_step": ms, "ms_per_step_mean": ms_mean,
            "step_ms": step_ms if world == 1 else None, "lanes_per_step": lanes_per_step,
@@ -522,10 +540,11 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     nd.load()
-    peak_flops = nd.measure_fp64_peak()
+    pipe_peak, pipe_src = fp64_pipe_peak(torch.cuda.get_device_properties(dev).multi_processor_count)
+    peaks = (pipe_peak, pipe_src, nd.measure_fp64_peak())
 
     progs, desc, B_total = population(args, args.config, world, rank, args.lanes)
-    head = measure(nd, dev, progs, B_total, args.config, args.dtype, args, world, rank, peak_flops, True)
+    head = measure(nd, dev, progs, B_total, args.config, args.dtype, args, world, rank, peaks, True)
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args, progs)
@@ -536,7 +555,7 @@ def main():
             if (cfg, dt) == (args.config, args.dtype):
                 continue
             p2, d2, bt2 = population(args, cfg, world, rank, 0)
-            m = measure(nd, dev, p2, bt2, cfg, dt, args, world, rank, peak_flops, False)
+            m = measure(nd, dev, p2, bt2, cfg, dt, args, world, rank, peaks, False)
             m["workload"] = f"{d2}, {dt} value+grad"
             if rank == 0 and not args.no_cpu_baseline:
                 m["cpu_baseline"] = bounded_cpu_baseline(p2, dt == "f32")

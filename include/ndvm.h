@@ -196,8 +196,10 @@ ndvm_status ndvm_tape_shared_work(const ndvm_tape* tape, double* work_per_call);
 
 /*
  * ndvm_measure_fp64_peak -- measure the device's FP64 fused multiply-add rate
- * (flop/s, two per FMA) with a dependent-chain microbenchmark on all SMs; the
- * roofline denominator for the replay, which is bound by FP64 issue.  Synchronous.
+ * (flop/s, two per FMA) with a dependent-chain microbenchmark on all SMs.  On GB300
+ * a saturated DFMA stream issues one warp instruction per 19 cycles per SM, 84 % of
+ * the FP64 pipe's unit-count peak (2 per clock per SM); the benchmark reports it
+ * beside that peak.  The paper has no counterpart.  Synchronous.
  */
 ndvm_status ndvm_measure_fp64_peak(double* flops_per_s, void* stream);
 

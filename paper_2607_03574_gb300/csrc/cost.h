@@ -1,20 +1,22 @@
-// Algorithmic FP64 work per tape primitive, in DFMA-equivalents (one fused
-// multiply-add issue of the FP64 pipe = 1).  Arithmetic counts one per add,
-// multiply or fused multiply-add; a first adjoint contribution that is a copy or a
-// sign flip counts zero.  Functions count their throughput cost relative to DFMA,
-// measured on GB300 with many independent calls per thread on finite arguments:
-// the replay's own exp 9.7 and log 12.6 (fmath.cuh), and CUDA's sin 17.1,
-// sincos 22.3, tanh 13.5, sqrt 7.3, division 7.1, reciprocal 4.4, log 28.5 (inside
-// pow's adjoint) and pow 79.9.  The roofline divides this work by the measured
-// DFMA rate.
+// Algorithmic FP64 work per tape primitive, in DFMA-equivalents (one FP64
+// instruction issue = 1).  Arithmetic counts one per add, multiply or fused
+// multiply-add; a first adjoint contribution that is a copy or a sign flip counts
+// zero.  A function counts the FP64 instructions one call executes on GB300, counted
+// by ncu (smsp__inst_executed_pipe_fp64 per call) on the cost probe
+// (ndvm_measure_op_cost: four independent chains per thread on every SM, finite
+// ordinary arguments), less the chain's one add: the replay's own exp 11 and log 13
+// (fmath.cuh), and CUDA's sin 18.25, sincos 23.25, tanh 24, sqrt 8, division 8,
+// reciprocal 5, log 29.75 (inside pow's adjoint) and pow 84.  Each call's device time
+// on the probe agrees with its instruction count within 5 %.  The roofline divides
+// this work by the FP64 pipe's peak issue rate.
 #pragma once
 #include "tape.h"
 
 namespace ndvm {
 namespace cost {
 
-constexpr double kExp = 9.7, kLog = 12.6, kSin = 17.1, kSinCos = 22.3, kTanh = 13.5, kSqrt = 7.3,
-                 kRcp = 4.4, kPow = 79.9, kDiv = 7.1, kLogLib = 28.5;
+constexpr double kExp = 11, kLog = 13, kSin = 18.25, kSinCos = 23.25, kTanh = 24, kSqrt = 8,
+                 kRcp = 5, kPow = 84, kDiv = 8, kLogLib = 29.75;
 
 inline double inv_cost(int n) {
   if (n == 1) return kDiv;
