@@ -1473,6 +1473,15 @@ Plan Planner::build() {
     pl.code.push_back(d);
   }
   for (const PArg& a : args_) pl.args.push_back(encode(a));
+  // one scratch area at the end of the slot file for the instructions that need working
+  // space beyond their operands (scratch_elems); each uses it only while it runs
+  int scratch = 0;
+  for (const DInst& d : pl.code) scratch = std::max(scratch, scratch_elems(d));
+  if (scratch > 0) {
+    for (DInst& d : pl.code)
+      if (scratch_elems(d) > 0) d.f[2] = mkref(RK_SLOT, pl.n_slots);
+    pl.n_slots += scratch;
+  }
   if (merge_loads_enabled()) pl.code = merge_obs_loads(pl.code);
   if (fma_enabled() && pair_enabled()) pl.code_paired = pair_fma(pl.code);
   for (const DInst& d : pl.code)
@@ -1490,6 +1499,14 @@ Plan Planner::build() {
 }
 
 }  // namespace
+
+int scratch_elems(const DInst& d) {
+  const int n = d.r;
+  if (d.op == B_INV) return n * n;
+  if (d.op == D_INV && n >= 4) return 2 * n * n;
+  if ((d.op == D_DET || d.op == D_LOGDET) && n >= 4) return (d.f[4] != -1 || d.f[5] >= 0) ? 2 * n * n : n * n;
+  return 0;
+}
 
 bool slot_operand(int op, int field) {
   switch (op) {
@@ -1547,6 +1564,11 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
     }
   };
   auto save_ok = [&](int32_t s, int64_t width) { return s == -1 || (s >= 0 && s + width <= p.n_save); };
+  // an instruction with working space names a slot area of its size (and none otherwise)
+  auto scratch_ok = [&](const DInst& d) {
+    const int need = scratch_elems(d);
+    return need == 0 ? d.f[2] == -1 : (d.f[2] != -1 && ref_ok(d.f[2], need, true));
+  };
   auto args_ok = [&](int32_t off, int64_t cnt, int stride) {
     return off >= 0 && cnt >= 0 && (size_t)off + (size_t)cnt * stride <= p.args.size();
   };
@@ -1589,11 +1611,12 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
         ok = ref_ok(f[0], w, true) && ref_ok(f[1], r * k, false) && ref_ok(f[2], k * c, false) && save_ok(f[3], w);
         break;
       case D_INV:
-        ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, false) && save_ok(f[3], n * n);
+        ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, false) && save_ok(f[3], n * n) &&
+             scratch_ok(d);
         break;
       case D_DET: case D_LOGDET:
         ok = n <= 8 && ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, false) && save_ok(f[3], 1) &&
-             ref_ok(f[4], n * n, true) && save_ok(f[5], n * n);
+             ref_ok(f[4], n * n, true) && save_ok(f[5], n * n) && scratch_ok(d);
         break;
       case D_TRACE: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, false); break;
       case D_ZERO: case D_GREDUCE: ok = f[1] >= 0 && ref_ok(f[0], f[1], true); break;
@@ -1652,7 +1675,9 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
         ok = ref_ok(f[0], w, true) && ref_ok(f[1], r * k, true) && ref_ok(f[2], k * c, true) && ref_ok(f[3], r * k, false) &&
              ref_ok(f[4], k * c, false);
         break;
-      case B_INV: ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, true) && ref_ok(f[5], n * n, false); break;
+      case B_INV:
+        ok = n <= 8 && ref_ok(f[0], n * n, true) && ref_ok(f[1], n * n, true) && ref_ok(f[5], n * n, false) && scratch_ok(d);
+        break;
       case B_DET: case B_LOGDET:
         ok = n <= 8 && ref_ok(f[0], 1, true) && ref_ok(f[1], n * n, true) && ref_ok(f[5], 1, false) && ref_ok(f[6], n * n, false);
         break;

@@ -36,8 +36,8 @@ enum DOp : uint8_t {
   D_MADD, D_MSUB,   // f0 out, f1 a, f2 b, f3 save; r x c
   D_MSCALE,         // f0 out, f1 s, f2 A, f3 save; r x c
   D_MATMUL,         // f0 out, f1 A, f2 B, f3 save; r x c, inner k
-  D_INV,            // f0 out, f1 A, f3 save; n = r
-  D_DET, D_LOGDET,  // f0 out, f1 A, f3 save, f4 aux slot (inverse), f5 aux save; n = r
+  D_INV,            // f0 out, f1 A, f2 scratch (n >= 4), f3 save; n = r
+  D_DET, D_LOGDET,  // f0 out, f1 A, f2 scratch (n >= 4), f3 save, f4 aux slot (inverse), f5 aux save; n = r
   D_TRACE,          // f0 out, f1 A; n = r
   // ---- data-axis regions ----
   D_ZERO,           // f0 slot, f1 count
@@ -65,7 +65,7 @@ enum DOp : uint8_t {
   B_MADD, B_MSUB,   // f1 ga, f2 gb; r x c
   B_MSCALE,         // f1 gs, f2 gA, f3 ps, f4 pA; r x c
   B_MATMUL,         // f1 gA, f2 gB, f3 pA, f4 pB; r x c, inner k
-  B_INV,            // f1 gA, f5 pz; n = r
+  B_INV,            // f1 gA, f2 scratch, f5 pz; n = r
   B_DET,            // f1 gA, f5 pz, f6 pinv; n = r
   B_LOGDET,         // f1 gA, f6 pinv; n = r
   B_TRACE,          // f1 gA; n = r
@@ -159,6 +159,11 @@ struct Plan {
   std::vector<DeriveInfo> derive_info;
   int64_t derived_elems = 0;
 };
+
+// Per-lane working space (slot elements) that an instruction needs beyond its operands,
+// named by its field f2: the inverse's adjoint keeps M = gZ B^T there (n^2); Gauss-Jordan
+// elimination (n >= 4) keeps [A | I] (2 n^2) or, for a determinant alone, A (n^2).
+int scratch_elems(const DInst& d);
 
 // Build the plan; throws BuildError on unsupported tapes.
 Plan make_plan(const Tape& t, bool grad, int force_mode = -1 /* -1 auto, 0 keep, 1 spill */);

@@ -44,36 +44,37 @@ struct Opnd {
   __device__ __forceinline__ const T* at(int e) const { return p + e * s; }
 };
 
-// a[0] b[0] + a[sa] b[sb] + ... over n terms, accumulated left to right with fma;
-// unrolled for n <= 8 so that all operand loads issue before the chain starts
+// s + a[0] b[0] + a[sa] b[sb] + ... over n terms, accumulated left to right with fma;
+// unrolled for n <= 8 so that all operand loads issue before the chain starts.  Started
+// from s = -0 it is the plain dot product (fma(a, b, -0) rounds a * b exactly as a
+// multiplication does, signed zeros included); started from an adjoint, the update
+// folds into the chain instead of costing a separate addition.
 template <typename T, int K>
-__device__ __forceinline__ T dot_fixed(const T* a, int sa, const T* b, int sb) {
+__device__ __forceinline__ T dot_fixed(const T* a, int sa, const T* b, int sb, T s) {
   T av[K], bv[K];
 #pragma unroll
   for (int q = 0; q < K; q++) { av[q] = a[q * sa]; bv[q] = b[q * sb]; }
-  T s = av[0] * bv[0];
 #pragma unroll
-  for (int q = 1; q < K; q++) s = fma(av[q], bv[q], s);
+  for (int q = 0; q < K; q++) s = fma(av[q], bv[q], s);
   return s;
 }
 template <typename T>
-__device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n) {
+__device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, T s) {
   switch (n) {
-    case 1: return a[0] * b[0];
-    case 2: return dot_fixed<T, 2>(a, sa, b, sb);
-    case 3: return dot_fixed<T, 3>(a, sa, b, sb);
-    case 4: return dot_fixed<T, 4>(a, sa, b, sb);
-    case 5: return dot_fixed<T, 5>(a, sa, b, sb);
-    case 6: return dot_fixed<T, 6>(a, sa, b, sb);
-    case 7: return dot_fixed<T, 7>(a, sa, b, sb);
-    case 8: return dot_fixed<T, 8>(a, sa, b, sb);
-    default: {
-      T s = a[0] * b[0];
-      for (int q = 1; q < n; q++) s = fma(a[q * sa], b[q * sb], s);
+    case 1: return fma(a[0], b[0], s);
+    case 2: return dot_fixed<T, 2>(a, sa, b, sb, s);
+    case 3: return dot_fixed<T, 3>(a, sa, b, sb, s);
+    case 4: return dot_fixed<T, 4>(a, sa, b, sb, s);
+    case 5: return dot_fixed<T, 5>(a, sa, b, sb, s);
+    case 6: return dot_fixed<T, 6>(a, sa, b, sb, s);
+    case 7: return dot_fixed<T, 7>(a, sa, b, sb, s);
+    case 8: return dot_fixed<T, 8>(a, sa, b, sb, s);
+    default:
+      for (int q = 0; q < n; q++) s = fma(a[q * sa], b[q * sb], s);
       return s;
-    }
   }
 }
+template <typename T> __device__ __forceinline__ T neg_zero() { return -(T)0; }
 
 // walks a thread's elements e = first, first + step, ... of a matrix with c columns
 // as (row, column) pairs without a division per element
@@ -133,6 +134,13 @@ struct Lane {
     T* q = wp(ref) + e * ss;
     *q = first ? v : *q + v;
   }
+  // adjoint update by a product a * b: the first contribution stores it (rounded as a
+  // multiplication); later ones fold it into the sum with one fused multiply-add
+  __device__ __forceinline__ void upd_fma(int32_t ref, int e, T a, T b, bool first) const {
+    if (!own(e)) return;
+    T* q = wp(ref) + e * ss;
+    *q = fma(a, b, first ? -(T)0 : *q);
+  }
   __device__ __forceinline__ void save_out(int32_t sidx, int e, T v) const {
     if (sidx >= 0 && own(e)) save[(int64_t)(sidx + e) * save_ld + col] = v;
   }
@@ -168,75 +176,102 @@ template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
   return z;
 }
 
-// determinant and (optionally) inverse of an n x n matrix read from an operand
-// (closed-form adjugate for n <= 3, Gauss-Jordan with partial pivoting above)
+// correctly rounded reciprocal: the value of the IEEE division 1 / x, at lower cost
+__device__ __forceinline__ double rcp_rn(double x) { return __drcp_rn(x); }
+__device__ __forceinline__ float rcp_rn(float x) { return __frcp_rn(x); }
+
+// Determinants and inverses to 3 x 3 in closed form, element by element: a lane's
+// thread group splits an inverse's elements like those of any other matrix result,
+// and every element has the same arithmetic whichever thread computes it.
+// cofactor of element (r, s) of a 3 x 3 matrix (the cyclic form carries the sign)
 template <typename T>
-__device__ T det_inv(const Opnd<T>& A, int n, T* inv /* n*n or nullptr */) {
-  if (n == 1) {
-    T d = A[0];
-    if (inv) inv[0] = (T)1 / d;
-    return d;
-  }
-  if (n == 2) {
-    T a0 = A[0], a1 = A[1], a2 = A[2], a3 = A[3];
-    T d = a0 * a3 - a1 * a2;
-    if (inv) {
-      T r = (T)1 / d;
-      inv[0] = a3 * r; inv[1] = -a1 * r; inv[2] = -a2 * r; inv[3] = a0 * r;
-    }
-    return d;
-  }
-  if (n == 3) {
-    T a[9];
-#pragma unroll
-    for (int i = 0; i < 9; i++) a[i] = A[i];
-    T c00 = a[4] * a[8] - a[5] * a[7];
-    T c01 = a[5] * a[6] - a[3] * a[8];
-    T c02 = a[3] * a[7] - a[4] * a[6];
-    T d = a[0] * c00 + a[1] * c01 + a[2] * c02;
-    if (inv) {
-      T c10 = a[2] * a[7] - a[1] * a[8];
-      T c11 = a[0] * a[8] - a[2] * a[6];
-      T c12 = a[1] * a[6] - a[0] * a[7];
-      T c20 = a[1] * a[5] - a[2] * a[4];
-      T c21 = a[2] * a[3] - a[0] * a[5];
-      T c22 = a[0] * a[4] - a[1] * a[3];
-      T r = (T)1 / d;
-      inv[0] = c00 * r; inv[1] = c10 * r; inv[2] = c20 * r;
-      inv[3] = c01 * r; inv[4] = c11 * r; inv[5] = c21 * r;
-      inv[6] = c02 * r; inv[7] = c12 * r; inv[8] = c22 * r;
-    }
-    return d;
-  }
-  // n = 4..8: elimination on [A | I] in thread-local memory
-  T w[8][16];
-  for (int i = 0; i < n; i++)
-    for (int j = 0; j < 2 * n; j++) w[i][j] = j < n ? A[i * n + j] : (T)(j - n == i ? 1 : 0);
+__device__ __forceinline__ T cof3(const Opnd<T>& A, int r, int s) {
+  const int r1 = r == 2 ? 0 : r + 1, r2 = r == 0 ? 2 : r - 1;
+  const int s1 = s == 2 ? 0 : s + 1, s2 = s == 0 ? 2 : s - 1;
+  return fma(A[r1 * 3 + s1], A[r2 * 3 + s2], -(A[r1 * 3 + s2] * A[r2 * 3 + s1]));
+}
+// determinant, n <= 3 (expansion along the first row)
+template <typename T>
+__device__ __forceinline__ T det_small(const Opnd<T>& A, int n) {
+  if (n == 1) return A[0];
+  if (n == 2) return fma(A[0], A[3], -(A[1] * A[2]));
+  return fma(A[2], cof3(A, 0, 2), fma(A[1], cof3(A, 0, 1), A[0] * cof3(A, 0, 0)));
+}
+// element e of the inverse, n <= 3, given r = 1 / det: the adjugate's element times r
+template <typename T>
+__device__ __forceinline__ T inv_small(const Opnd<T>& A, int n, int e, T r) {
+  if (n == 1) return r;
+  if (n == 2) return flip_sign(A[(e == 0 || e == 3) ? 3 - e : e], (unsigned)(e == 1 || e == 2)) * r;
+  const int i = e / 3, j = e - 3 * i;
+  return cof3(A, j, i) * r;
+}
+
+// IEEE bits of |x| as an integer: ordered like |x| for every value that is not a NaN
+__device__ __forceinline__ unsigned long long abs_key(double x) {
+  return (unsigned long long)__double_as_longlong(x) & 0x7fffffffffffffffULL;
+}
+__device__ __forceinline__ unsigned long long abs_key(float x) { return __float_as_uint(x) & 0x7fffffffu; }
+__device__ __forceinline__ bool nan_key(unsigned long long k, double) { return k > 0x7ff0000000000000ULL; }
+__device__ __forceinline__ bool nan_key(unsigned long long k, float) { return k > 0x7f800000ULL; }
+
+// Gauss-Jordan elimination with partial pivoting (n = 4..8) on [A | I] (want_inv) or on
+// A alone, in the lane's scratch slots at sref: n rows of wc = 2n (or n) elements,
+// row-major.  Rows are never moved: the exchanges are kept as a permutation in a
+// register, four bits per logical row, logical row i being physical row perm(i).  The
+// lane's threads split the columns: in a column step a thread normalizes the pivot row
+// in its own columns and eliminates the other rows there, so the only values the
+// threads share within a step are the pivot column's, which every thread reads before
+// any is written.  The pivot is the first logical row at or below the diagonal of
+// largest magnitude (a strict comparison; a NaN never wins), a row whose factor is
+// exactly zero is left alone, and every element takes the same operations as in the
+// sequential elimination.  Returns the determinant (the product of the pivots, negated
+// per exchange); the inverse's row i is physical row perm(i), columns n .. 2n-1.
+template <typename T, bool SYNC, typename LaneT>
+__device__ T gauss_jordan(const LaneT& L, const Opnd<T>& A, int n, int32_t sref, bool want_inv, uint32_t& perm) {
+  T* W = L.wp(sref);
+  const int ss = L.ss, wc = want_inv ? 2 * n : n;
+  const int first = L.first(), es = L.step();
+  for (int j = first; j < wc; j += es)
+    for (int i = 0; i < n; i++) W[(i * wc + j) * ss] = j < n ? A[i * n + j] : (T)(j - n == i ? 1 : 0);
+  perm = 0x76543210u;
+  if (SYNC) __syncwarp();
   T d = (T)1;
   for (int col = 0; col < n; col++) {
     int piv = col;
-    T best = fabs(w[col][col]);
-    for (int i = col + 1; i < n; i++)
-      if (fabs(w[i][col]) > best) { best = fabs(w[i][col]); piv = i; }
+    unsigned long long best = abs_key(W[((int)((perm >> (4 * col)) & 15u) * wc + col) * ss]);
+    for (int i = col + 1; i < n; i++) {
+      const unsigned long long k = abs_key(W[((int)((perm >> (4 * i)) & 15u) * wc + col) * ss]);
+      if (!nan_key(k, T()) && !nan_key(best, T()) && k > best) { best = k; piv = i; }
+    }
     if (piv != col) {
-      for (int j = 0; j < 2 * n; j++) { T t = w[col][j]; w[col][j] = w[piv][j]; w[piv][j] = t; }
+      const uint32_t a = (perm >> (4 * col)) & 15u, b = (perm >> (4 * piv)) & 15u;
+      perm = (perm & ~((15u << (4 * col)) | (15u << (4 * piv)))) | (b << (4 * col)) | (a << (4 * piv));
       d = -d;
     }
-    T pv = w[col][col];
+    const int pr = (int)((perm >> (4 * col)) & 15u);
+    const T pv = W[(pr * wc + col) * ss];
     d = d * pv;
-    T r = (T)1 / pv;
-    for (int j = 0; j < 2 * n; j++) w[col][j] = w[col][j] * r;
-    for (int i = 0; i < n; i++) {
-      if (i == col) continue;
-      T f = w[i][col];
-      if (f != (T)0)
-        for (int j = 0; j < 2 * n; j++) w[i][j] = w[i][j] - f * w[col][j];
+    const T r = rcp_rn(pv);
+    T fct[8];  // the pivot column in the other rows, by physical row
+#pragma unroll
+    for (int i = 0; i < 8; i++) fct[i] = (i < n && i != pr) ? W[(i * wc + col) * ss] : (T)0;
+    if (SYNC) __syncwarp();
+    for (int j = first; j < wc; j += es) {
+      const T p = W[(pr * wc + j) * ss] * r;
+      W[(pr * wc + j) * ss] = p;
+#pragma unroll
+      for (int i = 0; i < 8; i++)
+        if (i < n && i != pr && !is_zero(fct[i])) W[(i * wc + j) * ss] = fma(-fct[i], p, W[(i * wc + j) * ss]);
     }
+    if (SYNC) __syncwarp();
   }
-  if (inv)
-    for (int i = 0; i < n; i++)
-      for (int j = 0; j < n; j++) inv[i * n + j] = w[i][n + j];
   return d;
+}
+// element e = (i, j) of the inverse left by gauss_jordan in the scratch slots
+template <typename T, typename LaneT>
+__device__ __forceinline__ T gj_inverse(const LaneT& L, int32_t sref, int n, uint32_t perm, int e) {
+  const int i = e / n, j = e - i * n;
+  return L.wp(sref)[((int)((perm >> (4 * i)) & 15u) * 2 * n + n + j) * L.ss];
 }
 
 template <typename LaneT>
@@ -546,35 +581,47 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         const int c = in.c, kk = in.k;
         RowCol rc(L.first(), c);
         for (int e = L.first(); e < w; e += es, rc.next(es, c)) {
-          const T s = dot(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk);
+          const T s = dot(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk, neg_zero<T>());
           L.st(f[0], e, s);
           L.save_out(f[3], e, s);
         }
         break;
       }
       case D_INV: {
+        // each thread its own elements: closed forms to 3 x 3, else Gauss-Jordan
+        // elimination in the scratch slots (f2) shared by the lane's threads
         const int n = in.r;
-        T inv[64];
-        det_inv(L.rd(f[1]), n, inv);
+        Opnd<T> A = L.rd(f[1]);
+        uint32_t perm = 0;
+        T r = (T)0;
+        if (n <= 3) r = rcp_rn(det_small(A, n));
+        else gauss_jordan<T, SHARED>(L, A, n, f[2], true, perm);
         for (int e = L.first(); e < n * n; e += es) {
-          L.st(f[0], e, inv[e]);
-          L.save_out(f[3], e, inv[e]);
+          const T v = n <= 3 ? inv_small(A, n, e, r) : gj_inverse<T>(L, f[2], n, perm, e);
+          L.st(f[0], e, v);
+          L.save_out(f[3], e, v);
         }
         break;
       }
       case D_DET: case D_LOGDET: {
+        // with an auxiliary output (f4 slot / f5 save) the inverse comes too, for the
+        // reverse rule
         const int n = in.r;
         const bool aux = f[4] != -1 || f[5] >= 0;
-        T inv[64];
-        T dt = det_inv(L.rd(f[1]), n, aux ? inv : nullptr);
-        T z = in.op == D_DET ? dt : fast_log(dt);
+        Opnd<T> A = L.rd(f[1]);
+        uint32_t perm = 0;
+        const T dt = n <= 3 ? det_small(A, n) : gauss_jordan<T, SHARED>(L, A, n, f[2], aux, perm);
+        const T z = in.op == D_DET ? dt : fast_log(dt);
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
-        if (aux)
+        if (aux) {
+          const T r = n <= 3 ? rcp_rn(dt) : (T)0;
           for (int e = L.first(); e < n * n; e += es) {
-            if (f[4] != -1) L.st(f[4], e, inv[e]);
-            L.save_out(f[5], e, inv[e]);
+            const T v = n <= 3 ? inv_small(A, n, e, r) : gj_inverse<T>(L, f[2], n, perm, e);
+            if (f[4] != -1) L.st(f[4], e, v);
+            L.save_out(f[5], e, v);
           }
+        }
         break;
       }
       case D_TRACE: {
@@ -731,17 +778,18 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], w, fb); break; }
         if (f[1] != -1) {
           Opnd<T> A = L.rd(f[4]);
-          T s = L.sl(f[0], 0) * A[0];
-          for (int e = 1; e < w; e++) s = fma(L.sl(f[0], e), A[e], s);
-          L.upd(f[1], 0, s, fa);
+          T s = fa ? neg_zero<T>() : L.sl(f[1], 0);
+          for (int e = 0; e < w; e++) s = fma(L.sl(f[0], e), A[e], s);
+          L.st(f[1], 0, s);
         }
         if (f[2] != -1) {
           T s = L.ld(f[3]);
-          for (int e = L.first(); e < w; e += es) L.upd(f[2], e, s * L.sl(f[0], e), fb);
+          for (int e = L.first(); e < w; e += es) L.upd_fma(f[2], e, s, L.sl(f[0], e), fb);
         }
         break;
       }
       case B_MATMUL: {
+        // the running adjoint of each target element starts its dot product's chain
         const int r = in.r, c = in.c, kk = in.k;
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], r * kk, fa); zero_if_first(L, f[2], kk * c, fb); break; }
@@ -749,36 +797,40 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         if (f[1] != -1) {  // gA (r x k) += gZ (r x c) * B^T (B is k x c)
           Opnd<T> Bm = L.rd(f[4]);
           RowCol rq(L.first(), kk);
-          for (int e = L.first(); e < r * kk; e += es, rq.next(es, kk))
-            L.upd(f[1], e, dot(G_.at(rq.i * c), G_.s, Bm.at(rq.j * c), Bm.s, c), fa);
+          for (int e = L.first(); e < r * kk; e += es, rq.next(es, kk)) {
+            T* q = L.wp(f[1]) + e * L.ss;
+            *q = dot(G_.at(rq.i * c), G_.s, Bm.at(rq.j * c), Bm.s, c, fa ? neg_zero<T>() : *q);
+          }
         }
         if (f[2] != -1) {  // gB (k x c) += A^T (A is r x k) * gZ
           Opnd<T> A = L.rd(f[3]);
           RowCol qj(L.first(), c);
-          for (int e = L.first(); e < kk * c; e += es, qj.next(es, c))
-            L.upd(f[2], e, dot(A.at(qj.i), kk * A.s, G_.at(qj.j), c * G_.s, r), fb);
+          for (int e = L.first(); e < kk * c; e += es, qj.next(es, c)) {
+            T* q = L.wp(f[2]) + e * L.ss;
+            *q = dot(A.at(qj.i), kk * A.s, G_.at(qj.j), c * G_.s, r, fb ? neg_zero<T>() : *q);
+          }
         }
         break;
       }
       case B_INV: {
+        // gA -= B^T gZ B^T (B the inverse): M = gZ B^T into the scratch slots (f2), each
+        // thread its own elements, then each thread its own elements of gA from M
         const int n = in.r;
         bool fa = in.flags & 1;
         if (f[1] == -1) break;
         if (all_zero(L, f[0], n * n)) { zero_if_first(L, f[1], n * n, fa); break; }
         Opnd<T> Bv = L.rd(f[5]);
         Opnd<T> G_ = {L.wp(f[0]), L.ss};
-        T m[64];  // M = gZ B^T
-        for (int p = 0; p < n; p++)
-          for (int j = 0; j < n; j++) {
-            T s = G_[p * n] * Bv[j * n];
-            for (int q = 1; q < n; q++) s = fma(G_[p * n + q], Bv[j * n + q], s);
-            m[p * n + j] = s;
-          }
-        for (int e = L.first(); e < n * n; e += es) {  // gA -= B^T M
+        Opnd<T> M = {L.wp(f[2]), L.ss};
+        for (int e = L.first(); e < n * n; e += es) {
+          const int p = e / n, j = e - p * n;
+          L.wp(f[2])[e * L.ss] = dot(G_.at(p * n), G_.s, Bv.at(j * n), Bv.s, n, neg_zero<T>());
+        }
+        if (SHARED) __syncwarp();
+        for (int e = L.first(); e < n * n; e += es) {
           const int i = e / n, j = e - i * n;
-          T s = Bv[i] * m[j];
-          for (int p = 1; p < n; p++) s = fma(Bv[p * n + i], m[p * n + j], s);
-          L.upd(f[1], e, -s, fa);
+          T* q = L.wp(f[1]) + e * L.ss;
+          *q = -dot(Bv.at(i), n * Bv.s, M.at(j), n * M.s, n, fa ? neg_zero<T>() : -*q);
         }
         break;
       }
@@ -792,7 +844,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
         Opnd<T> Iv = L.rd(f[6]);
         for (int e = L.first(); e < n * n; e += es) {
           const int i = e / n, j = e - i * n;
-          L.upd(f[1], e, fac * Iv[j * n + i], fa);
+          L.upd_fma(f[1], e, fac, Iv[j * n + i], fa);
         }
         break;
       }
@@ -814,7 +866,7 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
           int32_t t = q[3 * e];
           bool first = q[3 * e + 1] != 0;
           if (is_zero(g)) zero_if_first(L, t, 1, first);
-          else L.upd(t, 0, g * L.sl(q[3 * e + 2], 0), first);
+          else L.upd_fma(t, 0, g, L.sl(q[3 * e + 2], 0), first);
         }
         break;
       }
