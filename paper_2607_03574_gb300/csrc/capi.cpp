@@ -222,7 +222,18 @@ Shape launch_shape(const Plan& p, size_t elem, int64_t B) {
     while (g < 16 && (size_t)p.n_slots * (128 / g + 1) * elem > kSmemLimit) g *= 2;
     s.log2g = ilog2(g);
     s.shared = 1;
-    s.sstride = 128 / g + 1;
+    // threads per block: the largest of 128, 64 and 32 whose grid spreads the lanes over
+    // the SMs within 5 % of the average (the busiest SM holds ceil(blocks / SMs) blocks);
+    // a 4-state filter's 8192 lanes in 16-lane blocks leave 56 SMs with 64 lanes and 96
+    // with 48, in 8-lane blocks 112 SMs with 56 and 40 with 48
+    auto spread = [&](int tpb) {
+      const int64_t lpb = tpb >> s.log2g;
+      const int64_t grid = (B + lpb - 1) / lpb;
+      return (double)((grid + sms - 1) / sms * lpb) * (double)sms / (double)B;
+    };
+    for (int t = 128; t >= 32 && t >= g; t /= 2)
+      if (spread(t) <= 1.05) { s.tpb = t; break; }
+    s.sstride = (s.tpb >> s.log2g) + 1;
     if ((size_t)p.n_slots * s.sstride * elem > kSmemLimit) {
       // block-cooperative: one lane per block, whose threads split every matrix
       // instruction (large state dimensions: the lane's slot file alone fills the block)
