@@ -40,6 +40,14 @@ bool fetch_trim_enabled() {
   return !(e && e[0] == '0');
 }
 
+// NDVM_FETCH_STRIDE=n (1..64) sets the instructions per prefetch window of the reverse
+// sweep (a tuning knob; default kFetchStride).
+int fetch_stride() {
+  const char* e = std::getenv("NDVM_FETCH_STRIDE");
+  const int v = e ? std::atoi(e) : 0;
+  return v >= 1 && v <= 64 ? v : kFetchStride;
+}
+
 // NDVM_DERIVE=0 computes the shared per-point values on every lane instead.
 bool derive_enabled() {
   const char* e = std::getenv("NDVM_DERIVE");
@@ -1266,14 +1274,15 @@ void Planner::prefetch_workspace() {
   if (rev_begin_ < 0) return;
   const int n = (int)code_.size();
   const int nins = n - rev_begin_;
-  const int nwin = (nins + kFetchStride - 1) / kFetchStride;
+  const int stride = fetch_stride();
+  const int nwin = (nins + stride - 1) / stride;
   std::vector<std::vector<std::pair<int, int>>> uses(nwin);  // window -> (pc, field)
   size_t total = 0;
   for (int pc = rev_begin_; pc < n; pc++) {
     const PInst& p = code_[pc];
     for (int fld = 0; fld < 8; fld++)
       if (slot_operand(p.d.op, fld) && p.f[fld].isref && p.f[fld].r.kind == RK_SAVE) {
-        uses[(pc - rev_begin_) / kFetchStride].push_back({pc, fld});
+        uses[(pc - rev_begin_) / stride].push_back({pc, fld});
         total++;
       }
   }
@@ -1331,7 +1340,7 @@ void Planner::prefetch_workspace() {
   for (int k = 0; k < kFetchWindows; k++) fetches(k, -1, out);  // prologue
   for (int k = 0; k < nwin; k++) {
     fetches(k + kFetchWindows, k, out);
-    for (int pc = rev_begin_ + k * kFetchStride; pc < std::min(n, rev_begin_ + (k + 1) * kFetchStride); pc++) {
+    for (int pc = rev_begin_ + k * stride; pc < std::min(n, rev_begin_ + (k + 1) * stride); pc++) {
       newpc[pc] = (int)out.size();
       out.push_back(code_[pc]);
     }

@@ -101,7 +101,7 @@ bool slot_operand(int op, int field);
 // ahead of use: the reverse sweep is cut into windows of kFetchStride instructions,
 // whose values are fetched kFetchWindows windows ahead, kFetchPairs per instruction.
 constexpr int kFetchPairs = 4;
-constexpr int kFetchStride = 4;
+constexpr int kFetchStride = 16;
 constexpr int kFetchWindows = 4;
 
 // "no save" in the 24-bit save fields of D_FMA2

@@ -379,16 +379,18 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
   // registers, and a shared-memory record is close at hand anyway)
   DInst nxt;
   if (!STAGED && a.n_code > 0) nxt = code[0];
+  int chunk_end = kStageChunk;  // staged: first instruction of the next chunk
   for (int pc = 0; pc < a.n_code; pc++) {
-    if (STAGED && pc > 0 && (pc % kStageChunk) == 0) {
+    if (STAGED && pc == chunk_end) {
       const int k = pc / kStageChunk;
       __syncthreads();  // every warp has left chunk k - 1: its buffer is free
       stage_copy(k + 1);
       asm volatile("cp.async.commit_group;\n" ::: "memory");
       asm volatile("cp.async.wait_group 1;\n" ::: "memory");  // chunk k has landed
       __syncthreads();
+      chunk_end += kStageChunk;
     }
-    const DInst in = STAGED ? stage[((pc / kStageChunk) & 1) * kStageChunk + pc % kStageChunk] : nxt;
+    const DInst in = STAGED ? stage[(unsigned)pc & (2 * kStageChunk - 1)] : nxt;
     if (!STAGED && pc + 1 < a.n_code) nxt = code[pc + 1];
 
     const int32_t* f = in.f;
