@@ -1075,7 +1075,8 @@ void Planner::normalize_operands() {
     if (p.d.op == D_ENDLOOP) p.f[0] = I(newpc[p.f[0].v]);
   }
   code_.swap(out);
-  if (rev_begin_ >= 0) rev_begin_ = newpc[rev_begin_];
+  // (a plan without a reverse sweep starts it one past its last instruction)
+  if (rev_begin_ >= 0) rev_begin_ = rev_begin_ < n ? newpc[rev_begin_] : (int)code_.size();
 }
 
 // A first adjoint contribution that is a plain copy needs no work when the new adjoint
