@@ -123,6 +123,37 @@ ndvm_status ndvm_value_and_grad(const ndvm_tape* tape, ndvm_dtype dtype, int64_t
                                 size_t ws_bytes, void* stream);
 
 /*
+ * ndvm_workspace_bytes_multi -- device workspace that ndvm_value_and_grad_multi needs
+ * for the batch (tapes[k] with B[k] lanes): per tape, its shared per-point values and
+ * all of its lanes' saved forward values, each tape's region 256-byte aligned.  0 when
+ * the batch needs none (or an argument is invalid).
+ */
+size_t ndvm_workspace_bytes_multi(const ndvm_tape* const* tapes, int32_t n_tapes, const int64_t* B,
+                                  ndvm_dtype dtype);
+
+/*
+ * ndvm_value_and_grad_multi -- ndvm_value_and_grad for a batch of tapes in as few
+ * launches as possible (the optional multi-tape extension of the boundary; the paper's
+ * setting of many candidate programs evaluated together, sections 5-6).  Tape k replays
+ * B[k] lanes with its own params[k] (device, B[k] x P_k), obs[k] (device, n_obs[k]
+ * values), loss[k] (device, B[k]) and grad[k] (device, B[k] x P_k); the results are
+ * those of n_tapes separate ndvm_value_and_grad calls.  Replays of the same kernel
+ * variant, block size, threads per lane and occupancy share one launch (up to 240
+ * tapes each); a batch with shared per-point values adds one launch of observation
+ * copies and one of derive plans in front.
+ *   tapes, B, params, obs, n_obs, loss, grad : host arrays of n_tapes entries
+ *   workspace : device, 256-byte aligned, at least ndvm_workspace_bytes_multi bytes
+ *               (NULL if that is 0); overwritten; not to be shared with a concurrent call
+ * Tapes with B[k] = 0 are skipped.  Returns NDVM_E_INVALID_ARG before any launch when an
+ * entry is invalid (the message names the tape) or the workspace is too small; the
+ * first call for a tape uploads it synchronously, as for ndvm_value_and_grad.
+ */
+ndvm_status ndvm_value_and_grad_multi(const ndvm_tape* const* tapes, int32_t n_tapes, ndvm_dtype dtype,
+                                      const int64_t* B, const void* const* params, const void* const* obs,
+                                      const int64_t* n_obs, void* const* loss, void* const* grad, void* workspace,
+                                      size_t ws_bytes, void* stream);
+
+/*
  * ndvm_value_and_grad_host -- the same computation through host buffers: copies
  * params and obs to the device, runs ndvm_value_and_grad, copies loss and grad
  * back, and synchronizes the stream.  Device buffers are cached per tape and

@@ -62,6 +62,8 @@ def load(build_if_missing: bool = True):
             "ndvm_workspace_bytes": (SZ, [P, I64, ctypes.c_int]),
             "ndvm_forward": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P]),
             "ndvm_value_and_grad": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P, SZ, P]),
+            "ndvm_workspace_bytes_multi": (SZ, [P, I32, P, ctypes.c_int]),
+            "ndvm_value_and_grad_multi": (ctypes.c_int, [P, I32, ctypes.c_int, P, P, P, P, P, P, P, SZ, P]),
             "ndvm_value_and_grad_host": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_value_and_grad_noalloc": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
             "ndvm_value_and_grad_host_async": (ctypes.c_int, [P, ctypes.c_int, I64, P, P, I64, P, P, P]),
@@ -271,6 +273,45 @@ def value_and_grad(tape: Tape, params, obs, loss=None, grad=None, workspace=None
                                       0 if obs is None else obs.numel(), _dev_ptr(loss, "loss"),
                                       _dev_ptr(grad, "grad"), _dev_ptr(workspace, "workspace"), nbytes,
                                       _stream_ptr(stream)))
+    return loss, grad
+
+
+def value_and_grad_multi(tapes, params, obs, loss=None, grad=None, workspace=None, stream=None):
+    """Loss and gradient of several tapes in one batched call (ndvm_value_and_grad_multi).
+    tapes: list of Tape; params[k]: (B_k, P_k) CUDA tensor; obs[k]: 1-d CUDA tensor (all of
+    one dtype).  Returns (losses, grads), lists of tensors.  Outputs and the default
+    workspace that this call allocates belong to `stream`."""
+    torch = _torch()
+    n = len(tapes)
+    if not (len(params) == len(obs) == n):
+        raise NdvmError(1, "tapes, params and obs must have the same length")
+    if n == 0:
+        return [], []
+    dt = _dtype_code(params[0])
+    for p in params:
+        if _dtype_code(p) != dt:
+            raise NdvmError(1, "every params tensor must have the same dtype")
+    with _on_stream(stream):
+        if loss is None:
+            loss = [torch.empty(p.shape[0], dtype=p.dtype, device=p.device) for p in params]
+        if grad is None:
+            grad = [torch.empty_like(p) for p in params]
+    Arr = ctypes.c_void_p * n
+    I64A = ctypes.c_int64 * n
+    th = Arr(*[t.handle for t in tapes])
+    B = I64A(*[p.shape[0] for p in params])
+    lib = load()
+    need = lib.ndvm_workspace_bytes_multi(th, n, B, dt)
+    if workspace is None:
+        key = (str(params[0].device), _stream_ptr(stream).value, "multi")
+        workspace = _default_ws.setdefault(key, Workspace()).get(need, params[0].device, stream)
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(lib.ndvm_value_and_grad_multi(
+        th, n, dt, B, Arr(*[_dev_ptr(p, "params").value for p in params]),
+        Arr(*[None if o is None else _dev_ptr(o, "obs").value for o in obs]),
+        I64A(*[0 if o is None else o.numel() for o in obs]),
+        Arr(*[_dev_ptr(l, "loss").value for l in loss]), Arr(*[_dev_ptr(g, "grad").value for g in grad]),
+        _dev_ptr(workspace, "workspace"), nbytes, _stream_ptr(stream)))
     return loss, grad
 
 

@@ -7,6 +7,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <map>
+#include <memory>
 #include <mutex>
 #include <new>
 #include <string>
@@ -405,6 +406,204 @@ ndvm_status run(ndvm_tape* t, bool grad, ndvm_dtype dtype, int64_t B, const void
   return NDVM_OK;
 }
 
+// resident blocks per SM of a launch shape (shared memory and registers)
+int resident_blocks(const Shape& s) {
+  const int by_smem = (int)(kSmemPerSm / (s.smem + kSmemPerBlockReserved));
+  const int regs = (s.shared || s.staged) ? kMaxRegsStagedOrShared : kMaxRegsPlain;
+  const int by_regs = kRegsPerSm / (regs * s.tpb);
+  return std::max(1, std::min(by_smem, by_regs));
+}
+
+// One replay of a batched launch: its arguments, its blocks and its launch shape.
+struct Member {
+  ReplayArgs a;
+  int64_t blocks;
+  Shape sh;
+};
+
+// Launches the members in as few kernels as possible: one per run of members with the
+// same kernel variant, block size, threads per lane and resident blocks per SM (so that
+// the launch's shared memory, its largest member's, costs no member its occupancy), at
+// most kMultiMax members and 2^31 - 1 blocks per launch.
+ndvm_status launch_members(std::vector<Member>& ms, bool f32, void* stream) {
+  auto key = [](const Member& m) {
+    return std::vector<int>{m.sh.shared, m.sh.staged, m.sh.log2g, m.sh.tpb, resident_blocks(m.sh)};
+  };
+  std::stable_sort(ms.begin(), ms.end(), [&](const Member& x, const Member& y) { return key(x) < key(y); });
+  std::unique_ptr<MultiArgs> table(new MultiArgs);  // about 31 KB: on the heap
+  for (size_t i = 0; i < ms.size();) {
+    MultiArgs& m = *table;
+    m.n = 0;
+    int64_t blocks = 0;
+    size_t smem = 0;
+    const std::vector<int> k = key(ms[i]);
+    while (i < ms.size() && m.n < kMultiMax && key(ms[i]) == k && blocks + ms[i].blocks <= 0x7fffffff) {
+      m.start[m.n] = (int)blocks;
+      m.a[m.n] = ms[i].a;
+      blocks += ms[i].blocks;
+      smem = std::max(smem, ms[i].sh.smem);
+      m.n++;
+      i++;
+    }
+    if (m.n == 0) return fail(NDVM_E_INVALID_ARG, "too many lanes for one launch");
+    m.start[m.n] = (int)blocks;
+    cudaError_t e;
+    {
+      std::lock_guard<std::mutex> lk(g_launch_mu);
+      e = launch_replay_multi(m, f32, (int)blocks, k[3], smem, (cudaStream_t)stream);
+      g_launches++;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "batched replay launch");
+  }
+  return NDVM_OK;
+}
+
+// Workspace of a batch: per tape with lanes, a 256-byte aligned region holding its
+// extended observations (shared per-point values) and then its lanes' saved values.
+// Returns the bytes needed; offsets[k] receives tape k's region (relative to the base).
+size_t multi_layout(ndvm_tape* const* tapes, int32_t n, const int64_t* B, size_t elem, std::vector<size_t>* offsets) {
+  size_t cur = 0;
+  for (int32_t k = 0; k < n; k++) {
+    size_t off = 0;
+    if (tapes[k] && B[k] > 0) {
+      const Plan& p = tapes[k]->grad_plan;
+      const size_t need = derived_bytes(p, elem) + (size_t)p.n_save * elem * (size_t)B[k];
+      if (need > 0) {
+        cur = (cur + 255) / 256 * 256;
+        off = cur;
+        cur += need;
+      }
+    }
+    if (offsets) offsets->push_back(off);
+  }
+  return cur;
+}
+
+ndvm_status run_multi(ndvm_tape* const* tapes, int32_t n, ndvm_dtype dtype, const int64_t* B,
+                      const void* const* params, const void* const* obs, const int64_t* n_obs, void* const* loss,
+                      void* const* grad, void* ws, size_t ws_bytes, void* stream) {
+  if (n < 0) return fail(NDVM_E_INVALID_ARG, "negative tape count");
+  if (n == 0) return NDVM_OK;
+  if (!tapes || !B || !params || !obs || !n_obs || !loss || !grad) return fail(NDVM_E_INVALID_ARG, "null argument array");
+  if (dtype != NDVM_F64 && dtype != NDVM_F32) return fail(NDVM_E_INVALID_ARG, "bad dtype");
+  if (ws && (reinterpret_cast<uintptr_t>(ws) & 255)) return fail(NDVM_E_INVALID_ARG, "workspace must be 256-byte aligned");
+  const size_t elem = dtype == NDVM_F32 ? sizeof(float) : sizeof(double);
+  for (int32_t k = 0; k < n; k++) {
+    const std::string at = " (tape " + std::to_string(k) + ")";
+    if (!tapes[k]) return fail(NDVM_E_INVALID_ARG, "null tape" + at);
+    if (B[k] < 0) return fail(NDVM_E_INVALID_ARG, "B must be >= 0" + at);
+    if (B[k] > (int64_t)1 << 40) return fail(NDVM_E_INVALID_ARG, "B too large" + at);
+    if (B[k] == 0) continue;
+    const Plan& p = tapes[k]->grad_plan;
+    if (p.n_params > 0 && (!params[k] || !grad[k])) return fail(NDVM_E_INVALID_ARG, "null params or grad" + at);
+    if (!loss[k]) return fail(NDVM_E_INVALID_ARG, "null loss" + at);
+    if (n_obs[k] < p.n_obs_min) return fail(NDVM_E_INVALID_ARG, "obs holds too few values" + at);
+    if (p.n_obs_min > 0 && !obs[k]) return fail(NDVM_E_INVALID_ARG, "null obs" + at);
+    if (launch_shape(p, elem, B[k]).smem > kSmemLimit)
+      return fail(NDVM_E_UNSUPPORTED, "tape needs more slots per lane than shared memory holds" + at);
+  }
+  std::vector<size_t> off;
+  const size_t need = multi_layout(tapes, n, B, elem, &off);
+  if (need > 0 && (!ws || ws_bytes < need))
+    return fail(NDVM_E_INVALID_ARG, "this batch needs a workspace of " + std::to_string(need) + " bytes");
+  std::vector<Member> main, der;
+  std::unique_ptr<CopyRuns> runs(new CopyRuns);
+  runs->n = 0;
+  std::vector<CopyRuns> run_batches;
+  for (int32_t k = 0; k < n; k++) {
+    if (B[k] == 0) continue;
+    ndvm_tape* t = tapes[k];
+    const Plan& p = t->grad_plan;
+    DevCache* dc = nullptr;
+    ndvm_status st = device_cache(t, &dc);
+    if (st != NDVM_OK) return st;
+    const DevPlan& dp = dc->grad;
+    char* base = static_cast<char*>(ws) + off[(size_t)k];
+    const size_t der_bytes = derived_bytes(p, elem);
+    if (der_bytes > 0) {
+      // the observations the program reads, then the derive plans (one lane per point)
+      if (p.n_obs_min > 0) {
+        if (runs->n == kCopyRunsMax) { run_batches.push_back(*runs); runs->n = 0; }
+        runs->src[runs->n] = obs[k];
+        runs->dst[runs->n] = base;
+        runs->words[runs->n] = (int64_t)((size_t)p.n_obs_min * elem / 4);
+        runs->n++;
+      }
+      for (size_t q = 0; q < p.derive.size(); q++) {
+        const Plan& dq = p.derive[q];
+        const DeriveInfo& di = p.derive_info[q];
+        const DevPlan& dd = dp.derive[q];
+        if (di.n_points <= 0) continue;
+        Member m;
+        m.sh = launch_shape(dq, elem, di.n_points);
+        ReplayArgs& a = m.a;
+        a.code = dd.code;
+        a.n_code = (int)dq.code.size();
+        a.args = dd.args;
+        a.consts = dtype == NDVM_F32 ? (const void*)dd.consts_f : (const void*)dd.consts_d;
+        a.obs = obs[k];
+        a.params = static_cast<const char*>(obs[k]) + (size_t)di.base * elem;
+        a.loss = nullptr;
+        a.grad = nullptr;
+        a.save = base + (size_t)(p.n_obs_min + di.offset) * elem;
+        a.save_ld = di.n_points;
+        a.P = (int)di.stride;
+        a.log2g = m.sh.log2g;
+        a.shared_lane = m.sh.shared;
+        a.sstride = m.sh.sstride;
+        a.staged = m.sh.staged;
+        a.stage_off = m.sh.stage_off;
+        a.err = dc->err;
+        a.lane0 = 0;
+        a.lane_end = di.n_points;
+        const int64_t lpb = m.sh.tpb >> m.sh.log2g;
+        m.blocks = (di.n_points + lpb - 1) / lpb;
+        der.push_back(m);
+      }
+    }
+    Member m;
+    m.sh = launch_shape(p, elem, B[k]);
+    ReplayArgs& a = m.a;
+    const bool paired = (m.sh.staged || m.sh.shared) && dp.code_paired != nullptr;
+    a.code = paired ? dp.code_paired : dp.code;
+    a.n_code = (int)(paired ? p.code_paired.size() : p.code.size());
+    a.args = dp.args;
+    a.consts = dtype == NDVM_F32 ? (const void*)dp.consts_f : (const void*)dp.consts_d;
+    a.obs = der_bytes > 0 ? (const void*)base : obs[k];
+    a.params = params[k];
+    a.loss = loss[k];
+    a.grad = grad[k];
+    a.save = base + der_bytes;
+    a.save_ld = B[k];
+    a.P = p.n_params;
+    a.log2g = m.sh.log2g;
+    a.shared_lane = m.sh.shared;
+    a.sstride = m.sh.sstride;
+    a.staged = m.sh.staged;
+    a.stage_off = m.sh.stage_off;
+    a.err = dc->err;
+    a.lane0 = 0;
+    a.lane_end = B[k];
+    const int64_t lpb = m.sh.tpb >> m.sh.log2g;
+    m.blocks = (B[k] + lpb - 1) / lpb;
+    if (m.blocks > 0x7fffffff) return fail(NDVM_E_INVALID_ARG, "too many lanes for one launch");
+    main.push_back(m);
+  }
+  if (runs->n > 0) run_batches.push_back(*runs);
+  for (const CopyRuns& c : run_batches) {
+    cudaError_t e;
+    {
+      std::lock_guard<std::mutex> lk(g_launch_mu);
+      e = launch_copy_runs(c, (cudaStream_t)stream);
+      g_launches++;
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "observation copies");
+  }
+  ndvm_status st = launch_members(der, dtype == NDVM_F32, stream);
+  if (st != NDVM_OK) return st;
+  return launch_members(main, dtype == NDVM_F32, stream);
+}
+
 ndvm_status ensure(void** buf, size_t* have, size_t need) {
   if (*have >= need && *buf) return NDVM_OK;
   cudaFree(*buf);
@@ -520,6 +719,22 @@ ndvm_status ndvm_value_and_grad(const ndvm_tape* tape, ndvm_dtype dtype, int64_t
                                 const void* obs, int64_t n_obs, void* loss, void* grad, void* ws, size_t ws_bytes,
                                 void* stream) {
   return run(const_cast<ndvm_tape*>(tape), true, dtype, B, params, obs, n_obs, loss, grad, ws, ws_bytes, stream);
+}
+
+size_t ndvm_workspace_bytes_multi(const ndvm_tape* const* tapes, int32_t n_tapes, const int64_t* B, ndvm_dtype dtype) {
+  if (!tapes || !B || n_tapes <= 0) return 0;
+  for (int32_t k = 0; k < n_tapes; k++)
+    if (B[k] < 0) return 0;
+  return multi_layout(const_cast<ndvm_tape* const*>(tapes), n_tapes, B, dtype == NDVM_F32 ? sizeof(float) : sizeof(double),
+                      nullptr);
+}
+
+ndvm_status ndvm_value_and_grad_multi(const ndvm_tape* const* tapes, int32_t n_tapes, ndvm_dtype dtype, const int64_t* B,
+                                      const void* const* params, const void* const* obs, const int64_t* n_obs,
+                                      void* const* loss, void* const* grad, void* workspace, size_t ws_bytes,
+                                      void* stream) {
+  return run_multi(const_cast<ndvm_tape* const*>(tapes), n_tapes, dtype, B, params, obs, n_obs, loss, grad, workspace,
+                   ws_bytes, stream);
 }
 
 }  // extern "C"

@@ -295,14 +295,14 @@ __device__ __forceinline__ void zero_if_first(const LaneT& L, int32_t ref, int w
 // the writes.  FP64 time is per warp instruction, so splitting matrix work keeps its
 // cost while G times more warps cover the lanes.
 template <typename T, bool SHARED, bool STAGED, bool BLOCK>
-__global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(ReplayArgs a) {
+__device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block) {
   static_assert(!BLOCK || SHARED, "a block-cooperative lane is an element-split group");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int tid = threadIdx.x;
   const int tpb = blockDim.x;
   const int G = 1 << a.log2g;
   const int lane_in_block = tid >> a.log2g;
-  const int64_t lane_raw = a.lane0 + (int64_t)blockIdx.x * (tpb >> a.log2g) + lane_in_block;
+  const int64_t lane_raw = a.lane0 + (int64_t)block * (tpb >> a.log2g) + lane_in_block;
   const int grank = tid & (G - 1);
   const bool live = lane_raw < a.lane_end;
   if (G == 1 && !live && !STAGED) return;  // staged blocks keep every thread for the block barriers
@@ -885,6 +885,67 @@ __global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(Repl
 }
 
 template <typename T, bool SHARED, bool STAGED, bool BLOCK>
+__global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay(ReplayArgs a) {
+  replay_body<T, SHARED, STAGED, BLOCK>(a, blockIdx.x);
+}
+
+// Several replays in one launch (one per tape of a batch, all of one kernel variant and
+// block size): block b serves the member m with start[m] <= b < start[m + 1], as its
+// block b - start[m].  The member table travels as the kernel's parameter.
+template <typename T, bool SHARED, bool STAGED, bool BLOCK>
+__global__ void __launch_bounds__(256, (SHARED || STAGED) ? 2 : 4) k_replay_multi(const __grid_constant__ MultiArgs ma) {
+  const int b = blockIdx.x;
+  int lo = 0, hi = ma.n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (ma.start[mid] <= b) lo = mid;
+    else hi = mid - 1;
+  }
+  replay_body<T, SHARED, STAGED, BLOCK>(ma.a[lo], b - ma.start[lo]);
+}
+
+template <typename T, bool SHARED, bool STAGED, bool BLOCK>
+cudaError_t launch_multi_v(const MultiArgs& m, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  static int configured_dev = -1;
+  static size_t configured_smem = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (configured_dev != dev || smem > configured_smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_replay_multi<T, SHARED, STAGED, BLOCK>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured_dev = dev;
+    configured_smem = smem;
+  }
+  k_replay_multi<T, SHARED, STAGED, BLOCK><<<blocks, tpb, smem, s>>>(m);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_multi_t(const MultiArgs& m, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  const ReplayArgs& a = m.a[0];  // every member has the same variant
+  if (a.shared_lane && (1 << a.log2g) > 32)
+    return a.staged ? launch_multi_v<T, true, true, true>(m, blocks, tpb, smem, s)
+                    : launch_multi_v<T, true, false, true>(m, blocks, tpb, smem, s);
+  if (a.shared_lane)
+    return a.staged ? launch_multi_v<T, true, true, false>(m, blocks, tpb, smem, s)
+                    : launch_multi_v<T, true, false, false>(m, blocks, tpb, smem, s);
+  return a.staged ? launch_multi_v<T, false, true, false>(m, blocks, tpb, smem, s)
+                  : launch_multi_v<T, false, false, false>(m, blocks, tpb, smem, s);
+}
+
+// Copies of n_copy runs of values (src[i] -> dst[i], len[i] elements of elem bytes, in
+// 4-byte words: every run's addresses and length are multiples of 4 bytes), one block
+// per run: the observations of a batch's tapes into their extended observation buffers.
+__global__ void __launch_bounds__(256) k_copy_runs(const __grid_constant__ CopyRuns c) {
+  const int r = blockIdx.x;
+  if (r >= c.n) return;
+  const uint32_t* src = static_cast<const uint32_t*>(c.src[r]);
+  uint32_t* dst = static_cast<uint32_t*>(c.dst[r]);
+  for (int64_t i = threadIdx.x; i < c.words[r]; i += blockDim.x) dst[i] = src[i];
+}
+
+template <typename T, bool SHARED, bool STAGED, bool BLOCK>
 cudaError_t launch_v(const ReplayArgs& a, int blocks, int tpb, size_t smem, cudaStream_t s) {
   static int configured_dev = -1;
   static size_t configured_smem = 0;
@@ -917,6 +978,17 @@ cudaError_t launch_t(const ReplayArgs& a, int blocks, int tpb, size_t smem, cuda
 
 cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s) {
   return f32 ? launch_t<float>(a, blocks, tpb, smem, s) : launch_t<double>(a, blocks, tpb, smem, s);
+}
+
+cudaError_t launch_replay_multi(const MultiArgs& m, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s) {
+  if (m.n < 1 || m.n > kMultiMax || blocks < 1) return cudaErrorInvalidValue;
+  return f32 ? launch_multi_t<float>(m, blocks, tpb, smem, s) : launch_multi_t<double>(m, blocks, tpb, smem, s);
+}
+
+cudaError_t launch_copy_runs(const CopyRuns& c, cudaStream_t s) {
+  if (c.n < 1 || c.n > kCopyRunsMax) return cudaErrorInvalidValue;
+  k_copy_runs<<<c.n, 256, 0, s>>>(c);
+  return cudaGetLastError();
 }
 
 }  // namespace ndvm

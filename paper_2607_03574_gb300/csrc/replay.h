@@ -32,6 +32,30 @@ struct ReplayArgs {
 
 cudaError_t launch_replay(const ReplayArgs& a, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
 
+// Replays of several tapes in one launch: member m takes blocks [start[m], start[m + 1]).
+// Every member has the same kernel variant (shared_lane, staged, threads per lane) and
+// block size; the launch's shared memory is the largest member's.  The table is the
+// kernel's parameter (at most 32 KB), so a launch holds at most kMultiMax members.
+constexpr int kMultiMax = 240;
+struct MultiArgs {
+  int n;
+  int start[kMultiMax + 1];
+  ReplayArgs a[kMultiMax];
+};
+static_assert(sizeof(MultiArgs) <= 32000, "kernel parameter space");
+cudaError_t launch_replay_multi(const MultiArgs& m, bool f32, int blocks, int tpb, size_t smem, cudaStream_t s);
+
+// Device-to-device copies of up to kCopyRunsMax runs of 4-byte words in one launch.
+constexpr int kCopyRunsMax = 1000;
+struct CopyRuns {
+  int n;
+  const void* src[kCopyRunsMax];
+  void* dst[kCopyRunsMax];
+  int64_t words[kCopyRunsMax];
+};
+static_assert(sizeof(CopyRuns) <= 32000, "kernel parameter space");
+cudaError_t launch_copy_runs(const CopyRuns& c, cudaStream_t s);
+
 // Instructions per staged chunk (two chunk buffers of 6 KB sit after the slot file).
 constexpr int kStageChunk = 128;
 
