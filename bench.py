@@ -7,7 +7,9 @@ forward and in reverse over B = 4096 parameter lanes and 256 data points (MSE lo
 region; L2 is flushed between timed steps.  Prints one JSON line: the headline
 configuration's numbers, and under "configs" the same measurement of every other
 configuration (exp-decay, logistic f64 and f32, the two Kalman filters, the 64-state
-population), each with a bounded CPU-oracle baseline.
+population), each with a bounded CPU-oracle baseline, and the 200 programs at 64 lanes
+each (launch-bound) timed both as one call per program on the streams and as one
+batched ndvm_value_and_grad_multi call.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
                     [--config C] [--dtype f32] [--only]
@@ -156,9 +158,10 @@ class ClockSampler:
 DEFAULT_LANES = {1: 64, 2: B_LANES, 3: 16384, 4: 8192, 5: 65536, 6: 1024}
 DESCRIPTIONS = {1: "exp-decay y = a exp(-b t) + c: {B} lanes x 50 points, MSE",
                 3: "logistic Euler (stack bytecode): {B} lanes x 1000 steps, 100 obs, MSE",
-                4: "4-state constant-velocity Kalman NLL: {B} lanes x 200 steps",
-                5: "8-state random stable Kalman NLL: {B} lanes x 1000 steps",
-                6: "64-state Kalman NLL population, 8-d observations: {B} lanes x 50 steps"}
+                4: "4-state constant-velocity Kalman NLL: {B} lanes x {T} steps",
+                5: "8-state random stable Kalman NLL: {B} lanes x {T} steps",
+                6: "64-state Kalman NLL population, 8-d observations: {B} lanes x {T} steps"}
+DEFAULT_T = {4: 200, 5: 1000, 6: 50}
 
 
 def population(args, cfg: int, world: int = 1, rank: int = 0, lanes_per_rank: int = 0):
@@ -176,8 +179,9 @@ def population(args, cfg: int, world: int = 1, rank: int = 0, lanes_per_rank: in
         progs = W.random_exprs(n_programs=args.programs, B=B_total, n_points=N_POINTS, seed=SEED)
         desc = (f"random-expression programs: {len(progs)} programs x {B_total} lanes x {N_POINTS} points, MSE")
     else:
-        progs = [W.config(cfg, B=B_total, seed=SEED)]
-        desc = DESCRIPTIONS[cfg].format(B=B_total)
+        T = (getattr(args, "T", 0) or DEFAULT_T[cfg]) if cfg in DEFAULT_T else None
+        progs = [W.config(cfg, B=B_total, seed=SEED, **({"T": T} if T else {}))]
+        desc = DESCRIPTIONS[cfg].format(B=B_total, T=T)
     lo, hi = lane_slice(B_total, world, rank)
     local = [replace(w, params=w.params[lo:hi]) for w in progs]
     return local, desc, B_total
@@ -298,12 +302,14 @@ def fp64_pipe_peak(sms: int) -> tuple[float, str]:
             f"({src}); ncu's FP64-pipe utilisation is relative to the same rate")
 
 
-def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks, want_gather):
+def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks, want_gather, batched=False):
     """Time one configuration: W warm-up steps, then K timed steps of a captured CUDA
     graph of one whole step (every program of this rank's slice), L2 flushed before
-    each; then the same work end to end through the host-buffer entry point.  Returns
-    the measurement and, on rank 0 when want_gather, the population gathered from every
-    rank's slice."""
+    each; then the same work end to end through the host-buffer entry point.  With
+    `batched`, one step is one ndvm_value_and_grad_multi call over every program (end to
+    end: pinned host copies in, the call, copies out) instead of one call per program on
+    the streams.  Returns the measurement and, on rank 0 when want_gather, the population
+    gathered from every rank's slice."""
     import torch
 
     tdt = torch.float32 if dtype == "f32" else torch.float64
@@ -332,6 +338,9 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks,
 
     def step():
         cur = torch.cuda.current_stream(dev)  # the capture stream while a graph is captured
+        if batched:
+            nd.value_and_grad_multi(tapes, params, obs, loss=loss, grad=grad, stream=cur)
+            return
         if n_streams <= 1:
             for k in range(len(tapes)):
                 nd.value_and_grad(tapes[k], params[k], obs[k], loss=loss[k], grad=grad[k], stream=cur)
@@ -415,7 +424,37 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks,
     hl = [torch.empty(w.B, dtype=tdt).pin_memory().numpy() for w in progs]
     hg = [torch.empty((w.B, w.P), dtype=tdt).pin_memory().numpy() for w in progs]
 
+    if batched:
+        # a batch caller's layout: every program's inputs packed in one pinned host buffer
+        # and one device buffer (per-program views), likewise the outputs, so that one
+        # copy moves each way
+        def packed(shapes):
+            n = sum(int(np.prod(sh)) for sh in shapes)
+            h = torch.empty(n, dtype=tdt).pin_memory()
+            d = torch.empty(n, dtype=tdt, device=dev)
+            views, off = [], 0
+            for sh in shapes:
+                m = int(np.prod(sh))
+                views.append((h[off:off + m].view(sh), d[off:off + m].view(sh)))
+                off += m
+            return h, d, views
+        hin, din, vin = packed([tuple(w.params.shape) for w in progs] + [tuple(w.obs.shape) for w in progs])
+        for (hv, _), a in zip(vin, [w.params for w in progs] + [w.obs for w in progs]):
+            hv.copy_(torch.from_numpy(np.ascontiguousarray(a, dtype=npdt)))
+        hout, dout, vout = packed([(w.B,) for w in progs] + [(w.B, w.P) for w in progs])
+        n_p = len(progs)
+        b_params, b_obs = [v[1] for v in vin[:n_p]], [v[1] for v in vin[n_p:]]
+        b_loss, b_grad = [v[1] for v in vout[:n_p]], [v[1] for v in vout[n_p:]]
+
     def e2e_step():
+        if batched:
+            # one copy in, one batched call, one copy out, on one stream, then one wait
+            cur = torch.cuda.current_stream(dev)
+            din.copy_(hin, non_blocking=True)
+            nd.value_and_grad_multi(tapes, b_params, b_obs, loss=b_loss, grad=b_grad, stream=cur)
+            hout.copy_(dout, non_blocking=True)
+            cur.synchronize()
+            return
         # every program's copies and replay queued on the streams, then one wait
         for k in range(len(tapes)):
             nd.value_and_grad_host_async(tapes[k], hp[k], ho[k], hl[k], hg[k], stream=side[k % len(side)])
@@ -440,7 +479,7 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks,
     roofline = {
         "bound": "alu", "achieved": achieved / 1e12, "peak": pipe_peak / 1e12, "unit": "TFLOP/s",
         "frac": max(t_fp64, t_hbm) / (ms * 1e-3),
-        "traffic": recorded_traffic(cfg, dtype, args.lanes, len(tapes)),
+        "traffic": recorded_traffic(cfg, dtype, args.lanes or args.T, len(tapes)),
         "peak_source": pipe_src,
         "peak_probe": probe_peak / 1e12, "frac_of_probe": achieved / probe_peak,
         "probe_source": "DFMA stream measured in this process (8 chains/thread, 4x256 threads/SM): "
@@ -472,6 +511,7 @@ def measure(nd, dev, local_progs, B_total, cfg, dtype, args, world, rank, peaks,
 
 
 EXTRA = [(1, "f64"), (3, "f64"), (3, "f32"), (4, "f64"), (5, "f64"), (6, "f64")]
+SMALL_LANES = 64  # lanes per program of the launch-bound batch measured both ways
 PROBE_ITERS = 2000
 
 
@@ -514,6 +554,8 @@ def main():
                          "every lane otherwise)")
     ap.add_argument("--lanes", type=int, default=0, help="lanes per program and rank instead of the "
                                                          "configuration's (smaller cases for profiling)")
+    ap.add_argument("--T", type=int, default=0, help="time steps of the Kalman configurations (4-6) instead of "
+                                                     "theirs (smaller cases for profiling)")
     ap.add_argument("--streams", type=int, default=16, help="CUDA streams the programs are spread over")
     ap.add_argument("--no-graph", dest="graph", action="store_false",
                     help="launch every step from the host instead of replaying a captured CUDA graph")
@@ -550,7 +592,7 @@ def main():
         cpu = cpu_baseline(args, progs)
 
     configs = {}
-    if not args.only and not args.lanes:
+    if not args.only and not args.lanes and not args.T:
         for cfg, dt in EXTRA:
             if (cfg, dt) == (args.config, args.dtype):
                 continue
@@ -560,6 +602,15 @@ def main():
             if rank == 0 and not args.no_cpu_baseline:
                 m["cpu_baseline"] = bounded_cpu_baseline(p2, dt == "f32")
             configs[f"{cfg}" if dt == "f64" else f"{cfg}_{dt}"] = m
+        # small populations (64 lanes per program), where launches dominate: one call per
+        # program on the streams against one batched call for all programs
+        p2, d2, bt2 = population(args, 2, world, rank, SMALL_LANES)
+        for key, bat in (("2_64lanes_streams", False), ("2_64lanes_batched", True)):
+            m = measure(nd, dev, p2, bt2, 2, "f64", args, world, rank, peaks, False, batched=bat)
+            m["workload"] = (f"{d2}, f64 value+grad, " +
+                             ("ndvm_value_and_grad_multi: one call for every program" if bat else
+                              f"one ndvm_value_and_grad call per program on {args.streams} streams"))
+            configs[key] = m
 
     if rank == 0:
         cfg_key = {"workload": f"{desc}, {args.dtype} value+grad", "programs": len(progs),
