@@ -17,25 +17,31 @@ namespace cost {
 
 constexpr double kExp = 11, kLog = 13, kSin = 18.25, kSinCos = 23.25, kTanh = 24, kSqrt = 8,
                  kRcp = 5, kPow = 84, kDiv = 8, kLogLib = 29.75;
+// A division a / b takes the correctly rounded reciprocal of b (kRcp) and one correction
+// step (a product and two fused multiply-adds): kRcp + kDivStep, the same as kDiv; its
+// reverse rule divides the adjoint by b with the forward sweep's reciprocal where the plan
+// keeps it (kDivStep), else again by the IEEE division (kDiv).
+constexpr double kDivStep = 3;
 
+// (the reciprocal of a determinant or pivot is the correctly rounded rcp)
 inline double inv_cost(int n) {
-  if (n == 1) return kDiv;
-  if (n == 2) return 2 + kDiv + 4;           // det, 1/det, four scaled cofactors
-  if (n == 3) return 18 + 3 + kDiv + 9;      // nine cofactors, det, 1/det, nine scalings
-  return 2.0 * n * n * n + n * kDiv;        // elimination
+  if (n == 1) return kRcp;
+  if (n == 2) return 2 + kRcp + 4;           // det, 1/det, four scaled cofactors
+  if (n == 3) return 18 + 3 + kRcp + 9;      // nine cofactors, det, 1/det, nine scalings
+  return 2.0 * n * n * n + n * kRcp;        // elimination
 }
 inline double det_cost(int n) {
   if (n == 1) return 0;
   if (n == 2) return 2;
   if (n == 3) return 9;
-  return (2.0 * n * n * n) / 3.0 + n * kDiv;
+  return (2.0 * n * n * n) / 3.0 + n * kRcp;
 }
 
 inline double fwd(int op, int r, int c, int imm, int n, bool with_aux) {
   const double e = (double)r * c;
   switch (op) {
     case OP_ADD: case OP_SUB: case OP_MUL: return 1;
-    case OP_DIV: return kDiv;
+    case OP_DIV: return kRcp + kDivStep;
     case OP_POW: return kPow;
     case OP_NEG: case OP_ABS: case OP_SELECT: return 0;
     case OP_EXP: return kExp;
@@ -63,7 +69,7 @@ inline double rev(int op, int r, int c, int imm, int n, bool aa, bool ba, bool a
     case OP_ADD: case OP_SUB: return acc(aa, a_init) + acc(ba, b_init);
     case OP_NEG: return acc(aa, a_init);
     case OP_MUL: return (aa ? 1 : 0) + (ba ? 1 : 0);
-    case OP_DIV: return kDiv + acc(aa, a_init) + (ba ? 1 : 0);
+    case OP_DIV: return (extra ? kDivStep : kDiv) + acc(aa, a_init) + (ba ? 1 : 0);  // extra: 1/b kept
     case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLogLib + 2 : 0);
     case OP_EXP: case OP_SIN: case OP_COS: case OP_ABS: return 1;
     case OP_TANH: return 2;

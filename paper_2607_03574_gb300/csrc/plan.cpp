@@ -351,7 +351,14 @@ void Planner::analyze() {
       auto need = [&](int x) { need_val_[x] = 1; };
       switch (n.op) {
         case OP_MUL: if (active_[n.a]) need(n.b); if (active_[n.b]) need(n.a); break;
-        case OP_DIV: if (active_[n.a]) need(n.b); if (active_[n.b]) { need(n.b); need(v); } break;
+        case OP_DIV:
+          // the reverse rule reads b and, inside a data-axis body (where it stays in a slot
+          // for the point's reverse sweep), the forward sweep's reciprocal of b; a lane-level
+          // division divides again (a workspace round trip for the reciprocal measured no
+          // faster on a serial chain)
+          need(n.b); if (active_[n.b]) need(v);
+          if (region_body_[v]) need_aux_[v] = 1;
+          break;
         case OP_POW: need(n.a); need(n.b); need(v); break;
         case OP_EXP: case OP_TANH: case OP_INV: need(v); break;
         case OP_LOG: case OP_ABS: case OP_POWI: need(n.a); break;
@@ -447,6 +454,14 @@ void Planner::emit_forward(int v) {
     case OP_ADD: case OP_SUB: case OP_MUL: case OP_DIV: case OP_POW:
       p.d.op = n.op == OP_ADD ? D_ADD : n.op == OP_SUB ? D_SUB : n.op == OP_MUL ? D_MUL : n.op == OP_DIV ? D_DIV : D_POW;
       p.f[1] = R(ref(n.a)); p.f[2] = R(ref(n.b)); p.f[3] = save_of(v);
+      if (n.op == OP_DIV && region_body_[v]) {
+        // through the correctly rounded reciprocal of b (flags bit 4), kept for the reverse rule
+        p.d.flags |= 16;
+        if (need_aux_[v]) {
+          if (aux_vr_[v] >= 0) p.f[4] = R(slotref(aux_vr_[v]));
+          else p.f[5] = I((int32_t)aux_save_[v]);
+        }
+      }
       break;
     case OP_NEG: case OP_EXP: case OP_LOG: case OP_TANH: case OP_SQRT: case OP_ABS:
       p.d.op = n.op == OP_NEG ? D_NEG : n.op == OP_EXP ? D_EXP : n.op == OP_LOG ? D_LOG : n.op == OP_TANH ? D_TANH
@@ -567,6 +582,7 @@ void Planner::emit_reverse(int v) {
       p.d.op = B_DIV; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
       p.f[4] = R(rref(n.b));
       if (active_[n.b]) p.f[5] = R(rref(v));
+      if (need_aux_[v]) p.f[6] = R(rauxref(v));
       break;
     case OP_POW:
       p.d.op = B_POW; tgt(n.a, 1, 0); tgt(n.b, 2, 1);
@@ -654,6 +670,7 @@ void Planner::emit_reverse(int v) {
     int extra = 0;
     if (n.op == OP_MATFROM) for (int k = 0; k < n.rows * n.cols; k++) extra += active_[T.args[n.imm + k]] ? 1 : 0;
     if (n.op == OP_DSUM) extra = (int)region_inputs_[v].size();
+    if (n.op == OP_DIV) extra = need_aux_[v] ? 1 : 0;  // the reverse rule has the reciprocal
     work_rev_ += mult_ * cost::rev(n.op, n.rows, n.cols, n.imm, in_rows, aa, ba, (flags & 1) != 0, (flags & 2) != 0, extra);
   }
   emit(p);
@@ -893,7 +910,7 @@ Plan Planner::build_derive(int r, const DeriveInfo& info) const {
       case OP_ADD: d.op = D_ADD; break;
       case OP_SUB: d.op = D_SUB; break;
       case OP_MUL: d.op = D_MUL; break;
-      case OP_DIV: d.op = D_DIV; break;
+      case OP_DIV: d.op = D_DIV; d.flags = 16; break;  // a body division: through 1/b, as in the replay
       case OP_POW: d.op = D_POW; break;
       case OP_NEG: d.op = D_NEG; break;
       case OP_EXP: d.op = D_EXP; break;
@@ -1096,7 +1113,7 @@ namespace {
 bool reads_only(int op, int fld) {
   if (op >= B_ADD && op <= B_GRAD) return fld == 0 || fld >= 3;  // gz and primal inputs; f1, f2 targets
   if (op == D_FETCH || fld == 0) return false;                    // destinations
-  if ((op == D_SIN || op == D_COS || op == D_DET || op == D_LOGDET) && fld == 4) return false;  // aux outputs
+  if ((op == D_SIN || op == D_COS || op == D_DET || op == D_LOGDET || op == D_DIV) && fld == 4) return false;  // aux outputs
   return true;
 }
 }  // namespace
@@ -1526,7 +1543,7 @@ bool slot_operand(int op, int field) {
       return field == 1;
     case D_SELECT: return field == 1 || field == 2 || field == 4;
     case B_MUL: return field == 3 || field == 4;
-    case B_DIV: return field == 4 || field == 5;
+    case B_DIV: return field == 4 || field == 5 || field == 6;
     case B_POW: return field == 3 || field == 4 || field == 5;
     case B_EXP: case B_TANH: return field == 5;
     case B_LOG: case B_ABS: case B_POWI: case B_SELECT: return field == 3;
@@ -1597,6 +1614,7 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
     switch (d.op) {
       case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: case D_CMP:
         ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && ref_ok(f[2], 1, false) && save_ok(f[3], 1);
+        if (d.op == D_DIV) ok = ok && ref_ok(f[4], 1, true) && save_ok(f[5], 1);  // the reciprocal of b
         break;
       case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: case D_POWI:
         ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, false) && save_ok(f[3], 1) && (d.op != D_POWI || (f[7] >= 0 && f[7] <= 64));
@@ -1662,7 +1680,7 @@ bool validate_code(const Plan& p, const std::vector<DInst>& code, size_t n_const
       case B_NEG: ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true); break;
       case B_MUL: case B_DIV: case B_POW:
         ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[2], 1, true) && ref_ok(f[3], 1, false) &&
-             ref_ok(f[4], 1, false) && ref_ok(f[5], 1, false);
+             ref_ok(f[4], 1, false) && ref_ok(f[5], 1, false) && (d.op != B_DIV || ref_ok(f[6], 1, false));
         break;
       case B_EXP: case B_TANH: case B_LOG: case B_ABS: case B_SQRT: case B_SIN: case B_COS: case B_POWI:
         ok = ref_ok(f[0], 1, true) && ref_ok(f[1], 1, true) && ref_ok(f[3], 1, false) && ref_ok(f[5], 1, false) &&

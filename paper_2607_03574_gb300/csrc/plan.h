@@ -26,7 +26,10 @@ inline int32_t ref_index(int32_t r) { return r & kRefIndexMask; }
 
 enum DOp : uint8_t {
   // ---- forward ----
-  D_ADD = 1, D_SUB, D_MUL, D_DIV, D_POW,  // f0 out, f1 a, f2 b, f3 save
+  D_ADD = 1, D_SUB, D_MUL, D_DIV, D_POW,  // f0 out, f1 a, f2 b, f3 save; D_DIV with flags bit 4 (a
+                    // division in a data-axis body): a / b by one correction step from 1/b correctly
+                    // rounded (the IEEE division outside the safe exponent range), 1/b kept in f4
+                    // aux slot / f5 aux save; without the bit, the IEEE division
   D_NEG, D_EXP, D_LOG, D_TANH, D_SQRT, D_ABS,  // f0 out, f1 a, f3 save
   D_SIN, D_COS,     // f0 out, f1 a, f3 save, f4 aux slot (the other trig value), f5 aux save
   D_POWI,           // f0 out, f1 a, f3 save, f7 n
@@ -51,7 +54,7 @@ enum DOp : uint8_t {
   //                     contribution to target 1/2, which stores instead of accumulating)
   B_ADD, B_SUB,     // f1 ga, f2 gb
   B_MUL,            // f1 ga, f2 gb, f3 pa, f4 pb
-  B_DIV,            // f1 ga, f2 gb, f4 pb, f5 pz
+  B_DIV,            // f1 ga, f2 gb, f4 pb, f5 pz, f6 p(1/b): g / b by one correction step from 1/b
   B_POW,            // f1 ga, f2 gb, f3 pa, f4 pb, f5 pz
   B_NEG,            // f1 ga
   B_EXP, B_TANH,    // f1 ga, f5 pz

@@ -180,6 +180,26 @@ template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
 __device__ __forceinline__ double rcp_rn(double x) { return __drcp_rn(x); }
 __device__ __forceinline__ float rcp_rn(float x) { return __frcp_rn(x); }
 
+// a / b from r, the correctly rounded reciprocal of b, by one correction step
+// (Markstein): q = a r, e = a - b q (exact by fma), q + r e.  The step is taken where a,
+// b and the quotient lie well inside the normal range (exponents within +-500 for double,
+// +-60 for float, zeros, infinities and NaNs excluded); elsewhere the IEEE division.
+__device__ __forceinline__ bool div_step_ok(double a, double b) {
+  const unsigned ea = (unsigned)(__double_as_longlong(a) >> 52) & 0x7ffu;
+  const unsigned eb = (unsigned)(__double_as_longlong(b) >> 52) & 0x7ffu;
+  return ea - 523u <= 1000u && eb - 523u <= 1000u;
+}
+__device__ __forceinline__ bool div_step_ok(float a, float b) {
+  const unsigned ea = (__float_as_uint(a) >> 23) & 0xffu, eb = (__float_as_uint(b) >> 23) & 0xffu;
+  return ea - 67u <= 120u && eb - 67u <= 120u;
+}
+template <typename T>
+__device__ __forceinline__ T div_by_rcp(T a, T b, T r) {
+  if (!div_step_ok(a, b)) return a / b;
+  const T q = a * r;
+  return fma(r, fma(-b, q, a), q);
+}
+
 // Determinants and inverses to 3 x 3 in closed form, element by element: a lane's
 // thread group splits an inverse's elements like those of any other matrix result,
 // and every element has the same arithmetic whichever thread computes it.
@@ -501,7 +521,6 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       NDVM_FWD2(D_ADD, x + y)
       NDVM_FWD2(D_SUB, x - y)
       NDVM_FWD2(D_MUL, x * y)
-      NDVM_FWD2(D_DIV, x / y)
       NDVM_FWD2(D_POW, pow(x, y))
       NDVM_FWD1(D_NEG, -x)
       NDVM_FWD1(D_EXP, fast_exp(x))
@@ -511,6 +530,25 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       NDVM_FWD1(D_ABS, fabs(x))
 #undef NDVM_FWD1
 #undef NDVM_FWD2
+      case D_DIV: {
+        // flags bit 4 (a division in a data-axis body): x / y through y's correctly rounded
+        // reciprocal, kept (f4 slot, f5 save) for the reverse rule, which divides its
+        // adjoint by y with it; else the IEEE division (staged streams have no data-axis
+        // bodies, so the staged variants carry the IEEE division alone)
+        const T x = L.lds(f[1]), y = L.lds(f[2]);
+        T z;
+        if (!STAGED && (in.flags & 16)) {
+          const T r = rcp_rn(y);
+          z = div_by_rcp(x, y, r);
+          if (f[4] != -1) L.st(f[4], 0, r);
+          L.save_out(f[5], 0, r);
+        } else {
+          z = x / y;
+        }
+        L.st(f[0], 0, z);
+        L.save_out(f[3], 0, z);
+        break;
+      }
       case D_SIN: case D_COS: {
         T x = L.lds(f[1]);
         T s = 0, c = 0;
@@ -701,7 +739,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         T g = L.sl(f[0], 0);
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
-        T q = g / L.lds(f[4]);
+        const T b = L.lds(f[4]);
+        const T q = f[6] != -1 ? div_by_rcp(g, b, L.lds(f[6])) : g / b;
         if (f[1] != -1) L.upd(f[1], 0, q, fa);
         if (f[2] != -1) L.upd(f[2], 0, -(q * L.lds(f[5])), fb);
         break;

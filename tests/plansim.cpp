@@ -33,6 +33,18 @@ namespace {
 
 bool is_zero(double x) { return x == 0.0; }
 bool gt_eps(double x) { return x > 1e-8; }
+// a / b from r = the correctly rounded 1 / b by one correction step where a and b have
+// exponents within +-500 (zeros, infinities and NaNs excluded), else the division
+double div_by_rcp(double a, double b, double r) {
+  int ea = 0, eb = 0;
+  std::frexp(a, &ea);
+  std::frexp(b, &eb);
+  const bool ok = std::isnormal(a) && std::isnormal(b) && ea - 1 >= -500 && ea - 1 <= 500 && eb - 1 >= -500 &&
+                  eb - 1 <= 500;
+  if (!ok) return a / b;
+  const double q = a * r;
+  return std::fma(r, std::fma(-b, q, a), q);
+}
 double powi_rep(double a, int n) {
   if (n == 0) return 1.0;
   double z = a;
@@ -217,10 +229,16 @@ struct Run {
           break;
         case D_ADD: case D_SUB: case D_MUL: case D_DIV: case D_POW: {
           const double x = ld(f[1]), y = ld(f[2]);
+          const double r = 1.0 / y;  // a body division (flags bit 4) keeps y's reciprocal
+          const bool via_rcp = in.op == D_DIV && (in.flags & 16);
           const double z = in.op == D_ADD ? x + y : in.op == D_SUB ? x - y : in.op == D_MUL ? x * y
-                           : in.op == D_DIV ? x / y : std::pow(x, y);
+                           : in.op == D_DIV ? (via_rcp ? div_by_rcp(x, y, r) : x / y) : std::pow(x, y);
           slot(f[0]) = z;
           save_out(f[3], z);
+          if (via_rcp) {
+            if (f[4] != -1) slot(f[4]) = r;
+            save_out(f[5], r);
+          }
           break;
         }
         case D_NEG: case D_EXP: case D_LOG: case D_TANH: case D_SQRT: case D_ABS: {
@@ -456,7 +474,7 @@ struct Run {
             if (f[1] != -1) upd(f[1], g * ld(f[4]), fa);
             if (f[2] != -1) upd(f[2], g * ld(f[3]), fb);
           } else if (in.op == B_DIV) {
-            const double q = g / ld(f[4]);
+            const double q = f[6] != -1 ? div_by_rcp(g, ld(f[4]), ld(f[6])) : g / ld(f[4]);
             if (f[1] != -1) upd(f[1], q, fa);
             if (f[2] != -1) upd(f[2], -(q * ld(f[5])), fb);
           } else {
