@@ -234,12 +234,14 @@ ndvm_status ndvm_tape_shared_work(const ndvm_tape* tape, double* work_per_call);
  */
 ndvm_status ndvm_measure_fp64_peak(double* flops_per_s, void* stream);
 
-/* Functions that ndvm_measure_op_cost times (the replay's own exp and log, CUDA's
- * other functions, and DFMA as the unit). */
+/* Functions that ndvm_measure_op_cost times (the replay's own exp, log, sin, cos and
+ * sincos; CUDA's other functions, and CUDA's log, exp, sin and sincos for comparison;
+ * DFMA as the unit). */
 enum {
   NDVM_PROBE_DFMA = 0, NDVM_PROBE_EXP = 1, NDVM_PROBE_LOG = 2, NDVM_PROBE_SIN = 3, NDVM_PROBE_COS = 4,
   NDVM_PROBE_SINCOS = 5, NDVM_PROBE_TANH = 6, NDVM_PROBE_SQRT = 7, NDVM_PROBE_DIV = 8, NDVM_PROBE_RCP = 9,
-  NDVM_PROBE_POW = 10, NDVM_PROBE_LOGLIB = 11, NDVM_PROBE_EXPLIB = 12, NDVM_PROBE_COUNT = 13
+  NDVM_PROBE_POW = 10, NDVM_PROBE_LOGLIB = 11, NDVM_PROBE_EXPLIB = 12, NDVM_PROBE_SINLIB = 13,
+  NDVM_PROBE_SINCOSLIB = 14, NDVM_PROBE_COUNT = 15
 };
 
 /*

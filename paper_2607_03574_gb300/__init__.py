@@ -163,7 +163,8 @@ def measure_fp64_peak(stream=None) -> float:
     return v.value
 
 
-PROBES = ("dfma", "exp", "log", "sin", "cos", "sincos", "tanh", "sqrt", "div", "rcp", "pow", "log_lib", "exp_lib")
+PROBES = ("dfma", "exp", "log", "sin", "cos", "sincos", "tanh", "sqrt", "div", "rcp", "pow", "log_lib", "exp_lib",
+          "sin_lib", "sincos_lib")
 
 
 def measure_op_cost(name: str, iters: int = 2000, stream=None) -> float:

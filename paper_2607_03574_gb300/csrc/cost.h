@@ -5,9 +5,11 @@
 // by ncu (smsp__inst_executed_pipe_fp64 per call) on the cost probe
 // (ndvm_measure_op_cost: four independent chains per thread on every SM, finite
 // ordinary arguments), less the chain's one add: the replay's own exp 11 and log 13
-// (fmath.cuh), and CUDA's sin 18.25, sincos 23.25, tanh 24, sqrt 8, division 8,
-// reciprocal 5, log 29.75 (inside pow's adjoint) and pow 84.  Each call's device time
-// on the probe agrees with its instruction count within 5 %.  The roofline divides
+// (fmath.cuh), and CUDA's tanh 24, sqrt 8, division 8, reciprocal 5, log 29.75 (inside
+// pow's adjoint) and pow 84.  Each call's device time on the probe agrees with its
+// instruction count within 5 %.  The replay's own sin (or cos) and sincos (fmath.cuh)
+// execute 16 and 19 FP64 instructions (counted in the source; the probe's device time
+// per call, 16.7 and 19.5 DFMA with the chain's add, agrees).  The roofline divides
 // this work by the FP64 pipe's peak issue rate.
 #pragma once
 #include "tape.h"
@@ -15,7 +17,7 @@
 namespace ndvm {
 namespace cost {
 
-constexpr double kExp = 11, kLog = 13, kSin = 18.25, kSinCos = 23.25, kTanh = 24, kSqrt = 8,
+constexpr double kExp = 11, kLog = 13, kSin = 16, kSinCos = 19, kTanh = 24, kSqrt = 8,
                  kRcp = 5, kPow = 84, kDiv = 8, kLogLib = 29.75;
 // A division a / b takes the correctly rounded reciprocal of b (kRcp) and one correction
 // step (a product and two fused multiply-adds): kRcp + kDivStep, the same as kDiv; its

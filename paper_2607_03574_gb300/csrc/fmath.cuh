@@ -16,8 +16,18 @@
 //   Taylor polynomial of log1p through u^7 (|u| <= 1/192; truncation < 2e-17
 //   relative).  For m near 1, F = 1 and the result is log1p(u) alone, so there is
 //   no cancellation.  13 FP64 instructions.
+// sin, cos: additive range reduction of W. J. Cody and W. Waite ("Software Manual for
+//   the Elementary Functions", 1980) by pi/64: x = n pi/64 + r, |r| <= pi/128, with pi/64
+//   in three parts (n times the first two exact for |n| < 2^20), then the addition
+//   formulas over a table of sin(k pi/64), k = n mod 128:
+//   sin x = S + (S (cos r - 1) + C sin r), cos x = C + (C (cos r - 1) - S sin r),
+//   S = sin(k pi/64), C = cos(k pi/64), with sin r through r^7 and cos r - 1 through r^6
+//   (truncation below 4e-19 relative at |r| = pi/128).  No branch on the quadrant: every
+//   lane of a warp runs the same instructions.  16 FP64 instructions for one of them, 19
+//   for both.
 // Arguments outside the fast range (|x| >= 708 for exp; x <= 0, subnormal, infinite
-// or NaN for log) take CUDA's exp / log.  Results are within about 1 ulp.
+// or NaN for log; |x| >= 2^15, infinite or NaN for sin and cos) take CUDA's functions.
+// Results are within about 1 ulp (sin and cos: 2 ulp, tested).
 #pragma once
 #include <cuda_runtime.h>
 
@@ -73,7 +83,49 @@ __device__ __forceinline__ double fast_log(double x) {
   return hi + lo;
 }
 
+// sin x and cos x; a caller that uses one of them leaves the other's instructions out
+__device__ __forceinline__ void fast_sincos(double x, double* s, double* c) {
+  const long long bx = __double_as_longlong(x);
+  if ((bx & 0x7fffffffffffffffLL) >= 0x40e0000000000000LL) {  // |x| >= 2^15, inf, nan
+    sincos(x, s, c);
+    return;
+  }
+  const double magic = 0x1.8p52;
+  const double t = fma(x, NDVM_64_PI, magic);
+  const int n = __double2loint(t);  // nearest integer to 64 x / pi
+  const double kd = t - magic;
+  double r = fma(kd, -NDVM_PI_64_1, x);
+  r = fma(kd, -NDVM_PI_64_2, r);
+  r = fma(kd, -NDVM_PI_64_3, r);
+  const double r2 = r * r;
+  double ps = fma(r2, -NDVM_INV5040, NDVM_INV120);
+  ps = fma(r2, ps, -NDVM_INV6);
+  const double sr = fma(r2 * r, ps, r);  // sin r
+  double pc = fma(r2, -NDVM_INV720, NDVM_INV24);
+  pc = fma(r2, pc, -0.5);
+  const double cm = r2 * pc;  // cos r - 1
+  const int k = n & 127;
+  const double S = kSinTable[k], C = kSinTable[(k + 32) & 127];
+  // |x| < 2^-27: sin x rounds to x and cos x to 1 (this also keeps the sign of a zero)
+  const bool tiny = (bx & 0x7fffffffffffffffLL) < 0x3e40000000000000LL;
+  *s = tiny ? x : S + fma(C, sr, S * cm);
+  *c = tiny ? 1.0 : C + fma(-S, sr, C * cm);
+}
+__device__ __forceinline__ double fast_sin(double x) {
+  double s, c;
+  fast_sincos(x, &s, &c);
+  return s;
+}
+__device__ __forceinline__ double fast_cos(double x) {
+  double s, c;
+  fast_sincos(x, &s, &c);
+  return c;
+}
+
 __device__ __forceinline__ float fast_exp(float x) { return expf(x); }
+__device__ __forceinline__ void fast_sincos(float x, float* s, float* c) { sincosf(x, s, c); }
+__device__ __forceinline__ float fast_sin(float x) { return sinf(x); }
+__device__ __forceinline__ float fast_cos(float x) { return cosf(x); }
 __device__ __forceinline__ float fast_log(float x) { return logf(x); }
 
 }  // namespace ndvm

@@ -553,14 +553,14 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         T x = L.lds(f[1]);
         T s = 0, c = 0;
         if (f[4] != -1 || f[5] >= 0) {
-          sincos(x, &s, &c);
+          fast_sincos(x, &s, &c);
           T aux = in.op == D_SIN ? c : s;
           if (f[4] != -1) L.st(f[4], 0, aux);
           L.save_out(f[5], 0, aux);
         } else if (in.op == D_SIN) {
-          s = sin(x);
+          s = fast_sin(x);
         } else {
-          c = cos(x);
+          c = fast_cos(x);
         }
         T z = in.op == D_SIN ? s : c;
         L.st(f[0], 0, z);
@@ -1102,9 +1102,11 @@ __device__ __forceinline__ double probe_f(double x) {
     case NDVM_PROBE_DFMA: return fma(x, 0.999999999, 1e-9);
     case NDVM_PROBE_EXP: return fast_exp(-x) + 0.25;
     case NDVM_PROBE_LOG: return fast_log(x) + 2.0;
-    case NDVM_PROBE_SIN: return sin(x) + 1.0;
-    case NDVM_PROBE_COS: return cos(x) + 1.0;
-    case NDVM_PROBE_SINCOS: { double s, c; sincos(x, &s, &c); return s + c; }
+    case NDVM_PROBE_SIN: return fast_sin(x) + 1.0;
+    case NDVM_PROBE_COS: return fast_cos(x) + 1.0;
+    case NDVM_PROBE_SINCOS: { double s, c; fast_sincos(x, &s, &c); return s + c; }
+    case NDVM_PROBE_SINLIB: return sin(x) + 1.0;
+    case NDVM_PROBE_SINCOSLIB: { double s, c; sincos(x, &s, &c); return s + c; }
     case NDVM_PROBE_TANH: return tanh(x) + 0.5;
     case NDVM_PROBE_SQRT: return sqrt(x) + 1.0;
     case NDVM_PROBE_DIV: return 3.0 / (x + 1.0);
@@ -1134,7 +1136,7 @@ using ProbeFn = void (*)(double*, int, int, cudaStream_t);
 constexpr ProbeFn kProbes[NDVM_PROBE_COUNT] = {
     launch_probe<0>, launch_probe<1>, launch_probe<2>, launch_probe<3>, launch_probe<4>,
     launch_probe<5>, launch_probe<6>, launch_probe<7>, launch_probe<8>, launch_probe<9>,
-    launch_probe<10>, launch_probe<11>, launch_probe<12>};
+    launch_probe<10>, launch_probe<11>, launch_probe<12>, launch_probe<13>, launch_probe<14>};
 }  // namespace
 
 cudaError_t measure_op_cost(int fn, int iters, double* ns_per_call, cudaStream_t s) {

@@ -1,5 +1,5 @@
-"""Accuracy of the replay's exp and log (GPU, through the C ABI) in units in the last
-place against the host's libm (numpy), over the full fast range and its edges."""
+"""Accuracy of the replay's exp, log, sin and cos (GPU, through the C ABI) in units in
+the last place against the host's libm (numpy), over the full fast range and its edges."""
 import numpy as np
 import pytest
 
@@ -50,3 +50,36 @@ def test_log_below_clamp_uses_the_clamp(ndvm, cuda):
     z, g = replay(ndvm, "(model (params a) (log a))", a)
     assert np.all(z == np.log(1e-8)) or ulps(z, np.full(5, np.log(1e-8))).max() <= 2.0
     np.testing.assert_array_equal(g, 0.0)
+
+
+def _trig_args(rng):
+    k = rng.integers(-20000, 20000, 20000)
+    return np.concatenate([
+        rng.uniform(-32767.0, 32767.0, 300000), rng.uniform(-10, 10, 200000), rng.uniform(-1e-8, 1e-8, 20000),
+        k * (np.pi / 2) + rng.uniform(-1e-6, 1e-6, 20000),  # near the zeros of sin and cos
+        k * (np.pi / 64) + rng.uniform(-np.pi / 128, np.pi / 128, 20000),  # around the table points
+        np.linspace(32766.0, 32769.0, 1001), -np.linspace(32766.0, 32769.0, 1001),  # the fast range's edge
+        [np.pi, -np.pi, np.pi / 2, 2 * np.pi, 1e5, -3e7, 1e300, 5e-324, np.inf, -np.inf, np.nan]])
+
+
+def _check_trig(z, ref):
+    fin = np.isfinite(ref)
+    assert np.array_equal(np.isnan(z), np.isnan(ref))
+    big = np.abs(ref[fin]) > 1e-300
+    assert ulps(z[fin][big], ref[fin][big]).max() <= 2.0
+
+
+def test_sin_cos_within_two_ulp(ndvm, cuda):
+    """sin (and its derivative, the cos that the forward sweep keeps) and cos."""
+    a = _trig_args(np.random.default_rng(7))
+    z, g = replay(ndvm, "(model (params a) (sin a))", a)
+    _check_trig(z, np.sin(a))
+    _check_trig(g, np.cos(a))
+    z, g = replay(ndvm, "(model (params a) (cos a))", a)
+    _check_trig(z, np.cos(a))
+    _check_trig(g, -np.sin(a))
+    # sin of a signed zero keeps its sign; cos of it is exactly 1
+    z, _ = replay(ndvm, "(model (params a) (sin a))", np.array([0.0, -0.0]))
+    assert np.array_equal(np.signbit(z), [False, True]) and np.all(z == 0.0)
+    z, _ = replay(ndvm, "(model (params a) (cos a))", np.array([0.0, -0.0]))
+    assert np.all(z == 1.0)
