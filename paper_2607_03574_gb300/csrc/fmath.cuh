@@ -35,9 +35,20 @@
 
 namespace ndvm {
 
+// The slow paths are calls, not inlined code: a rarely taken branch around inlined library
+// code can be compiled to predicated instructions that issue (all lanes off) every time,
+// and on GB300's FP64 pipe each of those costs a full slot.
+__device__ __noinline__ double slow_exp(double x) { return exp(x); }
+__device__ __noinline__ double slow_log(double x) { return log(x); }
+__device__ __noinline__ double2 slow_sincos(double x) {
+  double2 v;
+  sincos(x, &v.x, &v.y);
+  return v;
+}
+
 __device__ __forceinline__ double fast_exp(double x) {
   const long long bx = __double_as_longlong(x);
-  if ((bx & 0x7fffffffffffffffLL) >= 0x4086200000000000LL) return exp(x);  // |x| >= 708, inf, nan
+  if ((bx & 0x7fffffffffffffffLL) >= 0x4086200000000000LL) return slow_exp(x);  // |x| >= 708, inf, nan
   const double magic = 0x1.8p52;
   const double t = fma(x, NDVM_64_LN2, magic);
   const int n = __double2loint(t);  // nearest integer to 64 x / ln2
@@ -56,7 +67,7 @@ __device__ __forceinline__ double fast_exp(double x) {
 
 __device__ __forceinline__ double fast_log(double x) {
   const long long bx = __double_as_longlong(x);
-  if (bx < 0x0010000000000000LL || bx >= 0x7ff0000000000000LL) return log(x);  // <= 0, subnormal, inf, nan
+  if (bx < 0x0010000000000000LL || bx >= 0x7ff0000000000000LL) return slow_log(x);  // <= 0, subnormal, inf, nan
   int e = (int)(bx >> 52) - 1023;
   long long mb = (bx & 0x000fffffffffffffLL) | 0x3ff0000000000000LL;  // m in [1, 2)
   if (mb >= 0x3ff8000000000000LL) {  // m in [1.5, 2): use m/2 in [0.75, 1)
@@ -87,7 +98,9 @@ __device__ __forceinline__ double fast_log(double x) {
 __device__ __forceinline__ void fast_sincos(double x, double* s, double* c) {
   const long long bx = __double_as_longlong(x);
   if ((bx & 0x7fffffffffffffffLL) >= 0x40e0000000000000LL) {  // |x| >= 2^15, inf, nan
-    sincos(x, s, c);
+    const double2 v = slow_sincos(x);
+    *s = v.x;
+    *c = v.y;
     return;
   }
   const double magic = 0x1.8p52;

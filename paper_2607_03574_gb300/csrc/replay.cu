@@ -87,7 +87,10 @@ struct RowCol {
   }
 };
 
-template <typename T, bool SHARED>
+template <typename T> __device__ __noinline__ void add_to(T* q, T v) { *q = *q + v; }
+
+// BRANCH_ADD: accumulate through a call behind a real branch (see upd)
+template <typename T, bool SHARED, bool BRANCH_ADD>
 struct Lane {
   T* sbase;           // this thread's slot column: element s of the slot file is sbase[s * ss]
   int ss;             // slot row stride in elements
@@ -128,11 +131,18 @@ struct Lane {
   __device__ __forceinline__ void st(int32_t ref, int e, T v) const {
     if (own(e)) wp(ref)[e * ss] = v;
   }
-  // adjoint update: the first contribution stores, later ones accumulate
+  // adjoint update: the first contribution stores, later ones accumulate.  In the plain
+  // variant (BRANCH_ADD, the FP64-bound data-axis tapes) the accumulation is a call
+  // behind a real branch: inlined, the add is predicated and issues (all lanes off) on
+  // every first contribution, a full FP64 slot on GB300, and most targets of an
+  // expression tree get one contribution only; on a serial chain (the staged variant)
+  // the call's latency costs more than the slot
   __device__ __forceinline__ void upd(int32_t ref, int e, T v, bool first) const {
     if (!own(e)) return;
     T* q = wp(ref) + e * ss;
-    *q = first ? v : *q + v;
+    if (!BRANCH_ADD) *q = first ? v : *q + v;
+    else if (first) *q = v;
+    else add_to(q, v);
   }
   // adjoint update by a product a * b: the first contribution stores it (rounded as a
   // multiplication); later ones fold it into the sum with one fused multiply-add
@@ -169,11 +179,34 @@ __device__ __forceinline__ float flip_sign(float x, unsigned neg) {
   return __int_as_float(__float_as_int(x) ^ (int)(neg << 31));
 }
 
-template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
-  if (n == 0) return (T)1;
+// a^n by left-to-right repeated multiplication, and n a^(n-1) (the base adjoint of an
+// integer power): small n take straight-line code with literal factors (a loop with a
+// run-time trip count compiles to predicated multiplies, and converting n to a float
+// costs an FP64 slot); the same operations in the same order either way
+template <typename T> __device__ __forceinline__ T powi_loop(T a, int n) {
   T z = a;
+#pragma unroll 1
   for (int i = 1; i < n; i++) z = z * a;
   return z;
+}
+template <typename T> __device__ __forceinline__ T powi_rep(T a, int n) {
+  switch (n) {
+    case 0: return (T)1;
+    case 1: return a;
+    case 2: return a * a;
+    case 3: return (a * a) * a;
+    case 4: return ((a * a) * a) * a;
+    default: return powi_loop(a, n);
+  }
+}
+template <typename T> __device__ __forceinline__ T powi_deriv(T a, int n) {  // n >= 1
+  switch (n) {
+    case 1: return (T)1 * (T)1;
+    case 2: return (T)2 * a;
+    case 3: return (T)3 * (a * a);
+    case 4: return (T)4 * ((a * a) * a);
+    default: return (T)n * powi_loop(a, n - 1);
+  }
 }
 
 // correctly rounded reciprocal: the value of the IEEE division 1 / x, at lower cost
@@ -193,9 +226,49 @@ __device__ __forceinline__ bool div_step_ok(float a, float b) {
   const unsigned ea = (__float_as_uint(a) >> 23) & 0xffu, eb = (__float_as_uint(b) >> 23) & 0xffu;
   return ea - 67u <= 120u && eb - 67u <= 120u;
 }
+// the IEEE division and the correctly rounded reciprocal as calls (rarely taken paths;
+// see fmath.cuh's slow paths)
+template <typename T> __device__ __noinline__ T slow_div(T a, T b) { return a / b; }
+template <typename T> __device__ __noinline__ T slow_rcp(T b) { return rcp_rn(b); }
+
+// 1/b for b with an exponent within +-500 (div_step_ok): the hardware estimate
+// (rcp.approx.ftz.f64, off the FP64 pipe) refined by two Newton-Raphson steps
+// y <- y + y (1 - b y), each doubling its correct bits; 4 FP64 instructions and no
+// special-case code.  The result is within a hair of half an ulp, which is what the
+// correction step of a division needs.
+__device__ __forceinline__ double rcp_newton(double b) {
+  double y;
+  asm("rcp.approx.ftz.f64 %0, %1;" : "=d"(y) : "d"(b));
+  double e = fma(-b, y, 1.0);
+  y = fma(y, e, y);
+  e = fma(-b, y, 1.0);
+  return fma(y, e, y);
+}
+__device__ __forceinline__ float rcp_newton(float b) { return __frcp_rn(b); }
+
+// a / b and 1/b (into *r): in the safe range by the Newton reciprocal and one correction
+// step, else the IEEE division and the correctly rounded reciprocal
+template <typename T>
+__device__ __forceinline__ T div_rcp(T a, T b, T* r);
+template <typename T>
+__device__ __forceinline__ T div_rcp_q(T a, T b) {  // a / b alone
+  T r;
+  return div_rcp(a, b, &r);
+}
+template <typename T>
+__device__ __forceinline__ T div_rcp(T a, T b, T* r) {
+  if (!div_step_ok(a, b)) {
+    *r = slow_rcp(b);
+    return slow_div(a, b);
+  }
+  const T y = rcp_newton(b);
+  *r = y;
+  const T q = a * y;
+  return fma(y, fma(-b, q, a), q);
+}
 template <typename T>
 __device__ __forceinline__ T div_by_rcp(T a, T b, T r) {
-  if (!div_step_ok(a, b)) return a / b;
+  if (!div_step_ok(a, b)) return slow_div(a, b);
   const T q = a * r;
   return fma(r, fma(-b, q, a), q);
 }
@@ -327,7 +400,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
   const bool live = lane_raw < a.lane_end;
   if (G == 1 && !live && !STAGED) return;  // staged blocks keep every thread for the block barriers
 
-  Lane<T, SHARED> L;
+  Lane<T, SHARED, !SHARED && !STAGED> L;
   if (SHARED) {
     L.ss = a.sstride;
     L.sbase = reinterpret_cast<T*>(smem_raw) + lane_in_block;
@@ -538,12 +611,12 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         const T x = L.lds(f[1]), y = L.lds(f[2]);
         T z;
         if (!STAGED && (in.flags & 16)) {
-          const T r = rcp_rn(y);
-          z = div_by_rcp(x, y, r);
+          T r;
+          z = div_rcp(x, y, &r);
           if (f[4] != -1) L.st(f[4], 0, r);
           L.save_out(f[5], 0, r);
         } else {
-          z = x / y;
+          z = STAGED ? x / y : slow_div(x, y);  // a call where the other path is inlined
         }
         L.st(f[0], 0, z);
         L.save_out(f[3], 0, z);
@@ -740,7 +813,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         bool fa = in.flags & 1, fb = in.flags & 2;
         if (is_zero(g)) { zero_if_first(L, f[1], 1, fa); zero_if_first(L, f[2], 1, fb); break; }
         const T b = L.lds(f[4]);
-        const T q = f[6] != -1 ? div_by_rcp(g, b, L.lds(f[6])) : g / b;
+        const T q = f[6] != -1 ? div_by_rcp(g, b, L.lds(f[6])) : (STAGED ? g / b : slow_div(g, b));
         if (f[1] != -1) L.upd(f[1], 0, q, fa);
         if (f[2] != -1) L.upd(f[2], 0, -(q * L.lds(f[5])), fb);
         break;
@@ -766,12 +839,12 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
   }
       NDVM_REV1(B_EXP, g * L.lds(f[5]))
       NDVM_REV1(B_TANH, g * ((T)1 - L.lds(f[5]) * L.lds(f[5])))
-      NDVM_REV1(B_LOG, gt_eps(L.lds(f[3])) ? g / L.lds(f[3]) : (T)0)
+      NDVM_REV1(B_LOG, gt_eps(L.lds(f[3])) ? div_rcp_q(g, L.lds(f[3])) : (T)0)
       NDVM_REV1(B_ABS, L.lds(f[3]) > (T)0 ? g : (L.lds(f[3]) < (T)0 ? -g : g * (T)0))
       NDVM_REV1(B_SQRT, gt_eps(L.lds(f[3])) ? g / ((T)2 * L.lds(f[5])) : (T)0)
       NDVM_REV1(B_SIN, g * L.lds(f[6]))
       NDVM_REV1(B_COS, -(g * L.lds(f[6])))
-      NDVM_REV1(B_POWI, f[7] > 0 ? g * ((T)f[7] * powi_rep(L.lds(f[3]), f[7] - 1)) : (T)0)
+      NDVM_REV1(B_POWI, f[7] > 0 ? g * powi_deriv(L.lds(f[3]), f[7]) : (T)0)
 #undef NDVM_REV1
       case B_SELECT: {
         T g = L.sl(f[0], 0);
