@@ -19,11 +19,12 @@ namespace cost {
 
 constexpr double kExp = 11, kLog = 13, kSin = 16, kSinCos = 19, kTanh = 24, kSqrt = 8,
                  kRcp = 5, kPow = 84, kDiv = 8, kLogLib = 29.75;
-// A division a / b takes the correctly rounded reciprocal of b (kRcp) and one correction
-// step (a product and two fused multiply-adds): kRcp + kDivStep, the same as kDiv; its
-// reverse rule divides the adjoint by b with the forward sweep's reciprocal where the plan
-// keeps it (kDivStep), else again by the IEEE division (kDiv).
-constexpr double kDivStep = 3;
+// A division in a data-axis body takes 1/b from the hardware estimate and two Newton
+// steps (kRcpNewton: four fused multiply-adds) and one correction step (a product and
+// two fused multiply-adds, kDivStep); its reverse rule divides the adjoint by b with the
+// forward sweep's reciprocal (kDivStep).  A lane-level division is the IEEE division
+// (kDiv) in both sweeps.  The log's adjoint divides the same way as a body division.
+constexpr double kDivStep = 3, kRcpNewton = 4;
 
 // (the reciprocal of a determinant or pivot is the correctly rounded rcp)
 inline double inv_cost(int n) {
@@ -43,7 +44,7 @@ inline double fwd(int op, int r, int c, int imm, int n, bool with_aux) {
   const double e = (double)r * c;
   switch (op) {
     case OP_ADD: case OP_SUB: case OP_MUL: return 1;
-    case OP_DIV: return kRcp + kDivStep;
+    case OP_DIV: return with_aux ? kRcpNewton + kDivStep : kDiv;  // with_aux: a data-axis body
     case OP_POW: return kPow;
     case OP_NEG: case OP_ABS: case OP_SELECT: return 0;
     case OP_EXP: return kExp;
@@ -75,7 +76,7 @@ inline double rev(int op, int r, int c, int imm, int n, bool aa, bool ba, bool a
     case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLogLib + 2 : 0);
     case OP_EXP: case OP_SIN: case OP_COS: case OP_ABS: return 1;
     case OP_TANH: return 2;
-    case OP_LOG: return kDiv + 1;
+    case OP_LOG: return kRcpNewton + kDivStep + 1;
     case OP_SQRT: return kDiv + 2;
     case OP_POWI: return imm > 0 ? imm : 0;
     case OP_SELECT: return acc(aa, a_init) + acc(ba, b_init);

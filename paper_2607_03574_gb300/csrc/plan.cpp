@@ -448,7 +448,9 @@ void Planner::emit_forward(int v) {
   p.d.r = n.rows; p.d.c = n.cols;
   PRef out = slotref(val_vr_[v]);
   p.f[0] = R(out);
-  work_fwd_ += mult_ * cost::fwd(n.op, n.rows, n.cols, n.imm, T.nodes[n.a >= 0 ? n.a : v].rows, grad_ && need_aux_[v]);
+  // (with_aux: the auxiliary output is kept; for a division, that it runs in a data-axis body)
+  work_fwd_ += mult_ * cost::fwd(n.op, n.rows, n.cols, n.imm, T.nodes[n.a >= 0 ? n.a : v].rows,
+                                 n.op == OP_DIV ? region_body_[v] != 0 : grad_ && need_aux_[v]);
   nops_ += mult_;
   switch (n.op) {
     case OP_ADD: case OP_SUB: case OP_MUL: case OP_DIV: case OP_POW:
@@ -835,7 +837,7 @@ void Planner::plan_derived() {
     for (int u : cand) {
       if (used[u]) der_col_[u] = ncols++;
       const Node& m = T.nodes[u];
-      info.work += cost::fwd(m.op, 1, 1, m.imm, 1, false);
+      info.work += cost::fwd(m.op, 1, 1, m.imm, 1, m.op == OP_DIV);  // a derived division runs as a body division
     }
     info.n_cols = info.obs_cols + ncols;
     if ((int64_t)info.n_cols * info.n_points >= ((int64_t)1 << 27) ||
