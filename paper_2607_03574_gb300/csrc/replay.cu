@@ -44,6 +44,8 @@ struct Opnd {
   __device__ __forceinline__ const T* at(int e) const { return p + e * s; }
 };
 
+template <typename T> __device__ __forceinline__ T neg_zero() { return -(T)0; }
+
 // s + a[0] b[0] + a[sa] b[sb] + ... over n terms, accumulated left to right with fma;
 // unrolled for n <= 8 so that all operand loads issue before the chain starts.  Started
 // from s = -0 it is the plain dot product (fma(a, b, -0) rounds a * b exactly as a
@@ -69,12 +71,20 @@ __device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, 
     case 6: return dot_fixed<T, 6>(a, sa, b, sb, s);
     case 7: return dot_fixed<T, 7>(a, sa, b, sb, s);
     case 8: return dot_fixed<T, 8>(a, sa, b, sb, s);
-    default:
-      for (int q = 0; q < n; q++) s = fma(a[q * sa], b[q * sb], s);
-      return s;
+    default: {
+      // long products (n > 8): even and odd terms in two chains, joined at the end, so
+      // that each chain's dependent latency is half the product's
+      T s1 = neg_zero<T>();
+      int q = 0;
+      for (; q + 1 < n; q += 2) {
+        s = fma(a[q * sa], b[q * sb], s);
+        s1 = fma(a[(q + 1) * sa], b[(q + 1) * sb], s1);
+      }
+      if (q < n) s = fma(a[q * sa], b[q * sb], s);
+      return s + s1;
+    }
   }
 }
-template <typename T> __device__ __forceinline__ T neg_zero() { return -(T)0; }
 
 // walks a thread's elements e = first, first + step, ... of a matrix with c columns
 // as (row, column) pairs without a division per element
