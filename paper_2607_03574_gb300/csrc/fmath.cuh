@@ -1,6 +1,6 @@
 // Double-precision exp and log for the replay kernel, written for GB300's FP64
-// pipe: every FP64 instruction costs a 76-cycle issue slot of the shared FP64 unit
-// (1.675 fused multiply-adds per clock per SM), so range reduction, table indexing,
+// pipe: a warp's FP64 instruction occupies its scheduler's share of the FP64 unit for
+// 64 cycles (2 fused multiply-adds per clock per SM), so range reduction, table indexing,
 // exponent scaling and the special-case tests run on the integer pipes and the
 // FP64 pipe does only the arithmetic that needs 53-bit precision.
 //
@@ -35,6 +35,17 @@
 
 namespace ndvm {
 
+// The IEEE bits of x as an integer, through an inline-PTX move that the compiler's front
+// end cannot see through.  A test written on the bits of a computed double (x == +-0, a
+// range check) can otherwise be turned back into a floating-point compare, which runs on
+// the FP64 pipe and costs a full issue slot there; through fbits it stays on the integer
+// pipes.  The move itself is a register rename.
+__device__ __forceinline__ long long fbits(double x) {
+  long long b;
+  asm("mov.b64 %0, %1;" : "=l"(b) : "d"(x));
+  return b;
+}
+
 // The slow paths are calls, not inlined code: a rarely taken branch around inlined library
 // code can be compiled to predicated instructions that issue (all lanes off) every time,
 // and on GB300's FP64 pipe each of those costs a full slot.
@@ -47,7 +58,7 @@ __device__ __noinline__ double2 slow_sincos(double x) {
 }
 
 __device__ __forceinline__ double fast_exp(double x) {
-  const long long bx = __double_as_longlong(x);
+  const long long bx = fbits(x);
   if ((bx & 0x7fffffffffffffffLL) >= 0x4086200000000000LL) return slow_exp(x);  // |x| >= 708, inf, nan
   const double magic = 0x1.8p52;
   const double t = fma(x, NDVM_64_LN2, magic);
@@ -62,11 +73,11 @@ __device__ __forceinline__ double fast_exp(double x) {
   p = r * p;  // exp(r) - 1
   const double T = kExp2Table[n & 63];
   const double y = fma(T, p, T);
-  return __longlong_as_double(__double_as_longlong(y) + ((long long)(n >> 6) << 52));
+  return __longlong_as_double(fbits(y) + ((long long)(n >> 6) << 52));
 }
 
 __device__ __forceinline__ double fast_log(double x) {
-  const long long bx = __double_as_longlong(x);
+  const long long bx = fbits(x);
   if (bx < 0x0010000000000000LL || bx >= 0x7ff0000000000000LL) return slow_log(x);  // <= 0, subnormal, inf, nan
   int e = (int)(bx >> 52) - 1023;
   long long mb = (bx & 0x000fffffffffffffLL) | 0x3ff0000000000000LL;  // m in [1, 2)
@@ -96,7 +107,7 @@ __device__ __forceinline__ double fast_log(double x) {
 
 // sin x and cos x; a caller that uses one of them leaves the other's instructions out
 __device__ __forceinline__ void fast_sincos(double x, double* s, double* c) {
-  const long long bx = __double_as_longlong(x);
+  const long long bx = fbits(x);
   if ((bx & 0x7fffffffffffffffLL) >= 0x40e0000000000000LL) {  // |x| >= 2^15, inf, nan
     const double2 v = slow_sincos(x);
     *s = v.x;

@@ -169,11 +169,12 @@ struct Lane {
 template <typename T> __device__ __forceinline__ T clamp_eps() { return (T)1e-8; }
 
 // Tests on IEEE bit patterns run on the integer pipes, leaving the FP64 pipe to
-// arithmetic.  is_zero: +0 or -0.  gt_eps: x > 1e-8 with NaN false (IEEE order).
-__device__ __forceinline__ bool is_zero(double x) { return (__double_as_longlong(x) << 1) == 0; }
+// arithmetic (fbits keeps the compiler from turning them into FP64 compares).
+// is_zero: +0 or -0.  gt_eps: x > 1e-8 with NaN false (IEEE order).
+__device__ __forceinline__ bool is_zero(double x) { return (fbits(x) << 1) == 0; }
 __device__ __forceinline__ bool is_zero(float x) { return (__float_as_uint(x) << 1) == 0u; }
 __device__ __forceinline__ bool gt_eps(double x) {
-  const long long b = __double_as_longlong(x);
+  const long long b = fbits(x);
   return b > __double_as_longlong(1e-8) && (b & 0x7fffffffffffffffLL) <= 0x7ff0000000000000LL;
 }
 __device__ __forceinline__ bool gt_eps(float x) {
@@ -183,7 +184,7 @@ __device__ __forceinline__ bool gt_eps(float x) {
 
 // x with its sign bit flipped when neg is set (IEEE negation, exact for every value)
 __device__ __forceinline__ double flip_sign(double x, unsigned neg) {
-  return __longlong_as_double(__double_as_longlong(x) ^ ((long long)neg << 63));
+  return __longlong_as_double(fbits(x) ^ ((long long)neg << 63));
 }
 __device__ __forceinline__ float flip_sign(float x, unsigned neg) {
   return __int_as_float(__float_as_int(x) ^ (int)(neg << 31));
@@ -228,8 +229,8 @@ __device__ __forceinline__ float rcp_rn(float x) { return __frcp_rn(x); }
 // b and the quotient lie well inside the normal range (exponents within +-500 for double,
 // +-60 for float, zeros, infinities and NaNs excluded); elsewhere the IEEE division.
 __device__ __forceinline__ bool div_step_ok(double a, double b) {
-  const unsigned ea = (unsigned)(__double_as_longlong(a) >> 52) & 0x7ffu;
-  const unsigned eb = (unsigned)(__double_as_longlong(b) >> 52) & 0x7ffu;
+  const unsigned ea = (unsigned)(fbits(a) >> 52) & 0x7ffu;
+  const unsigned eb = (unsigned)(fbits(b) >> 52) & 0x7ffu;
   return ea - 523u <= 1000u && eb - 523u <= 1000u;
 }
 __device__ __forceinline__ bool div_step_ok(float a, float b) {
@@ -311,7 +312,7 @@ __device__ __forceinline__ T inv_small(const Opnd<T>& A, int n, int e, T r) {
 
 // IEEE bits of |x| as an integer: ordered like |x| for every value that is not a NaN
 __device__ __forceinline__ unsigned long long abs_key(double x) {
-  return (unsigned long long)__double_as_longlong(x) & 0x7fffffffffffffffULL;
+  return (unsigned long long)fbits(x) & 0x7fffffffffffffffULL;
 }
 __device__ __forceinline__ unsigned long long abs_key(float x) { return __float_as_uint(x) & 0x7fffffffu; }
 __device__ __forceinline__ bool nan_key(unsigned long long k, double) { return k > 0x7ff0000000000000ULL; }
