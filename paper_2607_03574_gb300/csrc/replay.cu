@@ -86,14 +86,37 @@ __device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, 
   }
 }
 
+// n / c for 0 <= n < 4096 and 1 <= c <= 255 without a division instruction (an integer
+// division by a run-time value compiles to a reciprocal sequence on the conversion and
+// special-function units): q = (n m) >> 20 with m = ceil(2^20 / c).  With
+// m c = 2^20 + d, 0 <= d < c, n m / 2^20 = n/c + n d / (c 2^20), and the excess stays
+// below 1/c, the least distance from n/c up to the next integer, while n c < 2^20.
+// Matrices are at most 64 x 64 (kMaxDim), so element indices stay below 4096, and
+// n m < 2^32.
+struct DivTable {
+  uint32_t m[256];
+  constexpr DivTable() : m() {
+    for (uint32_t c = 1; c < 256; c++) m[c] = ((1u << 20) + c - 1) / c;
+  }
+};
+__constant__ DivTable kDivTable = DivTable();
+__device__ __forceinline__ uint32_t div_magic(int c) { return kDivTable.m[c]; }
+__device__ __forceinline__ int divq(int n, uint32_t m) { return (int)(((uint32_t)n * m) >> 20); }
+
 // walks a thread's elements e = first, first + step, ... of a matrix with c columns
 // as (row, column) pairs without a division per element
 struct RowCol {
   int i, j;
-  __device__ __forceinline__ RowCol(int first, int c) : i(first / c), j(first - (first / c) * c) {}
+  uint32_t m;  // div_magic(c)
+  __device__ __forceinline__ RowCol(int first, int c) : m(div_magic(c)) {
+    i = divq(first, m);
+    j = first - i * c;
+  }
   __device__ __forceinline__ void next(int step, int c) {
     j += step;
-    while (j >= c) { j -= c; i++; }
+    const int q = divq(j, m);
+    i += q;
+    j -= q * c;
   }
 };
 
@@ -374,7 +397,7 @@ __device__ T gauss_jordan(const LaneT& L, const Opnd<T>& A, int n, int32_t sref,
 // element e = (i, j) of the inverse left by gauss_jordan in the scratch slots
 template <typename T, typename LaneT>
 __device__ __forceinline__ T gj_inverse(const LaneT& L, int32_t sref, int n, uint32_t perm, int e) {
-  const int i = e / n, j = e - i * n;
+  const int i = divq(e, div_magic(n)), j = e - i * n;
   return L.wp(sref)[((int)((perm >> (4 * i)) & 15u) * 2 * n + n + j) * L.ss];
 }
 
@@ -947,13 +970,14 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         Opnd<T> Bv = L.rd(f[5]);
         Opnd<T> G_ = {L.wp(f[0]), L.ss};
         Opnd<T> M = {L.wp(f[2]), L.ss};
+        const uint32_t mn = div_magic(n);
         for (int e = L.first(); e < n * n; e += es) {
-          const int p = e / n, j = e - p * n;
+          const int p = divq(e, mn), j = e - p * n;
           L.wp(f[2])[e * L.ss] = dot(G_.at(p * n), G_.s, Bv.at(j * n), Bv.s, n, neg_zero<T>());
         }
         if (SHARED) __syncwarp();
         for (int e = L.first(); e < n * n; e += es) {
-          const int i = e / n, j = e - i * n;
+          const int i = divq(e, mn), j = e - i * n;
           T* q = L.wp(f[1]) + e * L.ss;
           *q = -dot(Bv.at(i), n * Bv.s, M.at(j), n * M.s, n, fa ? neg_zero<T>() : -*q);
         }
@@ -967,8 +991,9 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         if (is_zero(g)) { zero_if_first(L, f[1], n * n, fa); break; }
         T fac = in.op == B_DET ? g * L.ld(f[5]) : g;
         Opnd<T> Iv = L.rd(f[6]);
+        const uint32_t mn = div_magic(n);
         for (int e = L.first(); e < n * n; e += es) {
-          const int i = e / n, j = e - i * n;
+          const int i = divq(e, mn), j = e - i * n;
           L.upd_fma(f[1], e, fac, Iv[j * n + i], fa);
         }
         break;
