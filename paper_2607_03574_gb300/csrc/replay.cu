@@ -171,21 +171,31 @@ struct Lane {
   // expression tree get one contribution only; on a serial chain (the staged variant)
   // the call's latency costs more than the slot
   __device__ __forceinline__ void upd(int32_t ref, int e, T v, bool first) const {
-    if (!own(e)) return;
+    if (own(e)) upd_mine(ref, e, v, first);
+  }
+  // adjoint update by a product a * b: the first contribution stores it (rounded as a
+  // multiplication); later ones fold it into the sum with one fused multiply-add
+  __device__ __forceinline__ void upd_fma(int32_t ref, int e, T a, T b, bool first) const {
+    if (own(e)) upd_fma_mine(ref, e, a, b, first);
+  }
+  __device__ __forceinline__ void save_out(int32_t sidx, int e, T v) const {
+    if (sidx >= 0 && own(e)) save[(int64_t)(sidx + e) * save_ld + col] = v;
+  }
+  // The element loops (e = first(), first() + step(), ...) visit only the thread's own
+  // elements: their writes skip the ownership test.
+  __device__ __forceinline__ void st_mine(int32_t ref, int e, T v) const { wp(ref)[e * ss] = v; }
+  __device__ __forceinline__ void save_mine(int32_t sidx, int e, T v) const {
+    if (sidx >= 0) save[(int64_t)(sidx + e) * save_ld + col] = v;
+  }
+  __device__ __forceinline__ void upd_mine(int32_t ref, int e, T v, bool first) const {
     T* q = wp(ref) + e * ss;
     if (!BRANCH_ADD) *q = first ? v : *q + v;
     else if (first) *q = v;
     else add_to(q, v);
   }
-  // adjoint update by a product a * b: the first contribution stores it (rounded as a
-  // multiplication); later ones fold it into the sum with one fused multiply-add
-  __device__ __forceinline__ void upd_fma(int32_t ref, int e, T a, T b, bool first) const {
-    if (!own(e)) return;
+  __device__ __forceinline__ void upd_fma_mine(int32_t ref, int e, T a, T b, bool first) const {
     T* q = wp(ref) + e * ss;
     *q = fma(a, b, first ? -(T)0 : *q);
-  }
-  __device__ __forceinline__ void save_out(int32_t sidx, int e, T v) const {
-    if (sidx >= 0 && own(e)) save[(int64_t)(sidx + e) * save_ld + col] = v;
   }
 };
 
@@ -541,10 +551,14 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       es = L.step();
     }
     if (in.op == D_FMA) {
-      // the fused form of the cheap scalar rules: no opcode dispatch
+      // the fused form of the cheap scalar rules: no opcode dispatch.  A zero gate (f4
+      // is +-0: a zero adjoint contributes nothing, even against an infinite factor)
+      // leaves c; it selects the inputs, fma(+0, -0, c) == c exactly for every c
+      // (signed zeros included), so no select waits on the multiply-add's result
       const T x = flip_sign(L.lds(f[1]), in.flags & 1);
       const T c = L.lds(f[3]);
-      const T z = is_zero(L.lds(f[4])) ? c : fma(x, L.lds(f[2]), c);
+      const bool off = is_zero(L.lds(f[4]));
+      const T z = fma(off ? (T)0 : x, off ? neg_zero<T>() : L.lds(f[2]), c);
       L.st(f[0], 0, z);
       L.save_out(f[5], 0, z);
       if (sync_each) group_sync();
@@ -557,7 +571,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       // (the plain variant is given the unpaired stream and does not carry this path)
       const T x1 = flip_sign(L.lds(f[1]), in.flags & 1), y1 = L.lds(f[2]), c1 = L.lds(f[3]), g1 = L.lds(f[4]);
       T x2 = L.lds(f[6]), y2 = L.lds(f[7]), c2 = L.lds(in.pad3), g2 = L.lds(in.pad4);
-      const T z1 = is_zero(g1) ? c1 : fma(x1, y1, c1);
+      const bool off1 = is_zero(g1);
+      const T z1 = fma(off1 ? (T)0 : x1, off1 ? neg_zero<T>() : y1, c1);
       if (in.flags & 4) {
         if (f[6] == f[0]) x2 = z1;
         if (f[7] == f[0]) y2 = z1;
@@ -565,7 +580,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         if (in.pad4 == f[0]) g2 = z1;
       }
       x2 = flip_sign(x2, (in.flags >> 1) & 1);
-      const T z2 = is_zero(g2) ? c2 : fma(x2, y2, c2);
+      const bool off2 = is_zero(g2);
+      const T z2 = fma(off2 ? (T)0 : x2, off2 ? neg_zero<T>() : y2, c2);
       L.st(f[0], 0, z1);
       L.st(f[5], 0, z2);
       if (in.flags & 8) {  // saves: 24-bit workspace indices in (r, c, k) and (pad0, pad1, pad2)
@@ -699,8 +715,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         const int32_t* g = args + f[1];
         for (int e = L.first(); e < f[2]; e += es) {
           T v = L.ld(g[e]);
-          L.st(f[0], e, v);
-          L.save_out(f[3], e, v);
+          L.st_mine(f[0], e, v);
+          L.save_mine(f[3], e, v);
         }
         break;
       }
@@ -708,8 +724,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         Opnd<T> A = L.rd(f[1]), Bm = L.rd(f[2]);
         for (int e = L.first(); e < w; e += es) {
           T z = in.op == D_MADD ? A[e] + Bm[e] : A[e] - Bm[e];
-          L.st(f[0], e, z);
-          L.save_out(f[3], e, z);
+          L.st_mine(f[0], e, z);
+          L.save_mine(f[3], e, z);
         }
         break;
       }
@@ -718,8 +734,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         Opnd<T> A = L.rd(f[2]);
         for (int e = L.first(); e < w; e += es) {
           T z = s * A[e];
-          L.st(f[0], e, z);
-          L.save_out(f[3], e, z);
+          L.st_mine(f[0], e, z);
+          L.save_mine(f[3], e, z);
         }
         break;
       }
@@ -729,8 +745,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         RowCol rc(L.first(), c);
         for (int e = L.first(); e < w; e += es, rc.next(es, c)) {
           const T s = dot(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk, neg_zero<T>());
-          L.st(f[0], e, s);
-          L.save_out(f[3], e, s);
+          L.st_mine(f[0], e, s);
+          L.save_mine(f[3], e, s);
         }
         break;
       }
@@ -745,8 +761,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         else gauss_jordan<T, SHARED>(L, A, n, f[2], true, perm);
         for (int e = L.first(); e < n * n; e += es) {
           const T v = n <= 3 ? inv_small(A, n, e, r) : gj_inverse<T>(L, f[2], n, perm, e);
-          L.st(f[0], e, v);
-          L.save_out(f[3], e, v);
+          L.st_mine(f[0], e, v);
+          L.save_mine(f[3], e, v);
         }
         break;
       }
@@ -765,8 +781,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
           const T r = n <= 3 ? rcp_rn(dt) : (T)0;
           for (int e = L.first(); e < n * n; e += es) {
             const T v = n <= 3 ? inv_small(A, n, e, r) : gj_inverse<T>(L, f[2], n, perm, e);
-            if (f[4] != -1) L.st(f[4], e, v);
-            L.save_out(f[5], e, v);
+            if (f[4] != -1) L.st_mine(f[4], e, v);
+            L.save_mine(f[5], e, v);
           }
         }
         break;
@@ -781,7 +797,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       }
       // ------------------------------------------------------------ data axis
       case D_ZERO:
-        for (int e = L.first(); e < f[1]; e += es) L.st(f[0], e, (T)0);
+        for (int e = L.first(); e < f[1]; e += es) L.st_mine(f[0], e, (T)0);
         break;
       case D_LOOP:
         dN = f[0]; dstride = f[1]; dbase0 = f[2];
@@ -916,8 +932,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         if (all_zero(L, f[0], w)) { zero_if_first(L, f[1], w, fa); zero_if_first(L, f[2], w, fb); break; }
         for (int e = L.first(); e < w; e += es) {
           T g = L.sl(f[0], e);
-          if (f[1] != -1) L.upd(f[1], e, g, fa);
-          if (f[2] != -1) L.upd(f[2], e, in.op == B_MADD ? g : -g, fb);
+          if (f[1] != -1) L.upd_mine(f[1], e, g, fa);
+          if (f[2] != -1) L.upd_mine(f[2], e, in.op == B_MADD ? g : -g, fb);
         }
         break;
       }
@@ -932,7 +948,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         }
         if (f[2] != -1) {
           T s = L.ld(f[3]);
-          for (int e = L.first(); e < w; e += es) L.upd_fma(f[2], e, s, L.sl(f[0], e), fb);
+          for (int e = L.first(); e < w; e += es) L.upd_fma_mine(f[2], e, s, L.sl(f[0], e), fb);
         }
         break;
       }
@@ -994,7 +1010,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         const uint32_t mn = div_magic(n);
         for (int e = L.first(); e < n * n; e += es) {
           const int i = divq(e, mn), j = e - i * n;
-          L.upd_fma(f[1], e, fac, Iv[j * n + i], fa);
+          L.upd_fma_mine(f[1], e, fac, Iv[j * n + i], fa);
         }
         break;
       }
