@@ -4,9 +4,10 @@
 // zero.  A function counts the FP64 instructions one call executes on GB300, counted
 // by ncu (smsp__inst_executed_pipe_fp64 per call) on the cost probe
 // (ndvm_measure_op_cost: four independent chains per thread on every SM, finite
-// ordinary arguments), less the chain's one add: the replay's own exp 11 and log 13
-// (fmath.cuh), and CUDA's tanh 24, sqrt 8, division 8, reciprocal 5, log 29.75 (inside
-// pow's adjoint) and pow 84.  Each call's device time on the probe agrees with its
+// ordinary arguments), less the chain's one add or multiply: the replay's own exp 10
+// and log 13 (fmath.cuh; the same counts in the source, and in ncu counts of
+// single-function programs through the replay), and CUDA's tanh 24, sqrt 8, division 8,
+// reciprocal 5, log 29.75 (inside pow's adjoint) and pow 84.  Each call's device time on the probe agrees with its
 // instruction count within 5 %.  The replay's own sin (or cos) and sincos (fmath.cuh)
 // execute 16 and 19 FP64 instructions (counted in the source; the probe's device time
 // per call, 16.7 and 19.5 DFMA with the chain's add, agrees).  The roofline divides
@@ -17,7 +18,7 @@
 namespace ndvm {
 namespace cost {
 
-constexpr double kExp = 11, kLog = 13, kSin = 16, kSinCos = 19, kTanh = 24, kSqrt = 8,
+constexpr double kExp = 10, kLog = 13, kSin = 16, kSinCos = 19, kTanh = 24, kSqrt = 8,
                  kRcp = 5, kPow = 84, kDiv = 8, kLogLib = 29.75;
 // A division in a data-axis body takes 1/b from the hardware estimate and two Newton
 // steps (kRcpNewton: four fused multiply-adds) and one correction step (a product and
@@ -76,8 +77,8 @@ inline double rev(int op, int r, int c, int imm, int n, bool aa, bool ba, bool a
     case OP_POW: return (aa ? kDiv + 2 : 0) + (ba ? kLogLib + 2 : 0);
     case OP_EXP: case OP_SIN: case OP_COS: case OP_ABS: return 1;
     case OP_TANH: return 2;
-    case OP_LOG: return kRcpNewton + kDivStep + 1;
-    case OP_SQRT: return kDiv + 2;
+    case OP_LOG: return kRcpNewton + kDivStep + acc(aa, a_init);  // g / x
+    case OP_SQRT: return kDiv + 1 + acc(aa, a_init);             // g / (2 z)
     case OP_POWI: return imm > 0 ? imm : 0;
     case OP_SELECT: return acc(aa, a_init) + acc(ba, b_init);
     case OP_MATFROM: return 0.0 + extra * 0.5;  // scattered copies and adds

@@ -1214,9 +1214,9 @@ cudaError_t measure_fp64_peak(double* flops_per_s, cudaStream_t s) {
 // ---------------------------------------------------------------------------
 // Per-function cost probe: the throughput of one library function (or of the
 // replay's own exp and log) relative to DFMA, for the roofline's cost table.  Every
-// thread runs four independent chains x <- f(x) + c (c keeps x in the function's
-// ordinary domain); one FP64 add per call is part of the chain and is counted in the
-// measured time.  Launch shape and iteration count match the FP64 peak probe's
+// thread runs four independent chains x <- f(x) + c (or f(x) c; c keeps x in the
+// function's ordinary domain); one FP64 add or multiply per call is part of the chain
+// and is counted in the measured time.  Launch shape and iteration count match the FP64 peak probe's
 // per-thread work, so an ncu capture of a probe launch gives the function's FP64-pipe
 // instructions per call (calls = blocks x threads x iters x 4).
 namespace ndvm {
@@ -1225,7 +1225,7 @@ template <int FN>
 __device__ __forceinline__ double probe_f(double x) {
   switch (FN) {
     case NDVM_PROBE_DFMA: return fma(x, 0.999999999, 1e-9);
-    case NDVM_PROBE_EXP: return fast_exp(-x) + 0.25;
+    case NDVM_PROBE_EXP: return fast_exp(x) * 0.25;  // x settles near 0.357
     case NDVM_PROBE_LOG: return fast_log(x) + 2.0;
     case NDVM_PROBE_SIN: return fast_sin(x) + 1.0;
     case NDVM_PROBE_COS: return fast_cos(x) + 1.0;
@@ -1238,7 +1238,7 @@ __device__ __forceinline__ double probe_f(double x) {
     case NDVM_PROBE_RCP: return 1.0 / x + 0.5;
     case NDVM_PROBE_POW: return pow(x, 0.75) + 1.0;
     case NDVM_PROBE_LOGLIB: return log(x) + 2.0;
-    case NDVM_PROBE_EXPLIB: return exp(-x) + 0.25;
+    case NDVM_PROBE_EXPLIB: return exp(x) * 0.25;
     default: return x;
   }
 }
