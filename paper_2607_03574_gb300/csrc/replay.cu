@@ -550,7 +550,11 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       L.emask = wide ? G - 1 : 31;
       es = L.step();
     }
-    if (in.op == D_FMA) {
+    // The fused scalar records and the fetches: ahead of the opcode switch where they make
+    // up most of the stream (scalar tapes), as switch cases in the element-split variants,
+    // whose streams are mostly matrix instructions
+    constexpr bool kFastFirst = !SHARED;
+    auto op_fma = [&]() {
       // the fused form of the cheap scalar rules: no opcode dispatch.  A zero gate (f4
       // is +-0: a zero adjoint contributes nothing, even against an infinite factor)
       // leaves c; it selects the inputs, fma(+0, -0, c) == c exactly for every c
@@ -561,10 +565,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       const T z = fma(off ? (T)0 : x, off ? neg_zero<T>() : L.lds(f[2]), c);
       L.st(f[0], 0, z);
       L.save_out(f[5], 0, z);
-      if (sync_each) group_sync();
-      continue;
-    }
-    if ((SHARED || STAGED) && in.op == D_FMA2) {
+    };
+    auto op_fma2 = [&]() {
       // two fused updates in one record: every operand is loaded before either store;
       // when the second reads the first's result (flags bit 2), the operands that name
       // the first's destination take its value from the register instead
@@ -589,10 +591,8 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         if (s1 != kNoSave24) L.save_out(s1, 0, z1);
         if (s2 != kNoSave24) L.save_out(s2, 0, z2);
       }
-      if (sync_each) group_sync();
-      continue;
-    }
-    if (in.op == D_FETCH) {
+    };
+    auto op_fetch = [&]() {
       // asynchronous copies of workspace values into slots (the owner of element 0
       // copies; the warp barrier after the wait publishes them to the group)
       // (unrolled: the record's fields stay in registers only when indexed by constants)
@@ -618,8 +618,23 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
           default: asm volatile("cp.async.wait_group %0;\n" ::"n"(kFetchWindows) : "memory"); break;
         }
       }
-      if (sync_each) group_sync();
-      continue;
+    };
+    if (kFastFirst) {
+      if (in.op == D_FMA) {
+        op_fma();
+        if (sync_each) group_sync();
+        continue;
+      }
+      if (STAGED && in.op == D_FMA2) {
+        op_fma2();
+        if (sync_each) group_sync();
+        continue;
+      }
+      if (in.op == D_FETCH) {
+        op_fetch();
+        if (sync_each) group_sync();
+        continue;
+      }
     }
     const int w = in.r * in.c;
     switch (in.op) {
@@ -1038,6 +1053,19 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
       }
       case B_GRAD:
         if (writer) grad[L.lane * L.P + f[1]] = f[0] == -1 ? (T)0 : L.sl(f[0], 0);
+        break;
+      case D_FMA:
+        if (!kFastFirst) op_fma();
+        break;
+      case D_FMA2:
+        if (!kFastFirst) {
+          op_fma2();
+          break;
+        }
+        if (a.err) atomicExch(a.err, 1);  // the plain variant carries no paired records
+        return;
+      case D_FETCH:
+        if (!kFastFirst) op_fetch();
         break;
       default:  // not an opcode of this variant: every thread stops
         if (a.err) atomicExch(a.err, 1);
