@@ -74,8 +74,20 @@ __device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, 
     default: {
       // long products (n > 8): even and odd terms in two chains, joined at the end, so
       // that each chain's dependent latency is half the product's
+      // (eight terms at a time with every load issued first; the even and odd terms keep
+      // their chains, so the sums are the same to the last bit)
       T s1 = neg_zero<T>();
       int q = 0;
+      for (; q + 8 <= n; q += 8) {
+        T av[8], bv[8];
+#pragma unroll
+        for (int u = 0; u < 8; u++) { av[u] = a[(q + u) * sa]; bv[u] = b[(q + u) * sb]; }
+#pragma unroll
+        for (int u = 0; u < 8; u += 2) {
+          s = fma(av[u], bv[u], s);
+          s1 = fma(av[u + 1], bv[u + 1], s1);
+        }
+      }
       for (; q + 1 < n; q += 2) {
         s = fma(a[q * sa], b[q * sb], s);
         s1 = fma(a[(q + 1) * sa], b[(q + 1) * sb], s1);
