@@ -60,7 +60,10 @@ __device__ __forceinline__ T dot_fixed(const T* a, int sa, const T* b, int sb, T
   for (int q = 0; q < K; q++) s = fma(av[q], bv[q], s);
   return s;
 }
-template <typename T>
+// WIDE: the long products' eight-term blocks (the element-split variants, whose matrices
+// reach 64 x 64); the other variants keep the two-term loop and its smaller register
+// footprint.  Both sum the same terms in the same chains.
+template <typename T, bool WIDE = true>
 __device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, T s) {
   switch (n) {
     case 1: return fma(a[0], b[0], s);
@@ -78,7 +81,7 @@ __device__ __forceinline__ T dot(const T* a, int sa, const T* b, int sb, int n, 
       // their chains, so the sums are the same to the last bit)
       T s1 = neg_zero<T>();
       int q = 0;
-      for (; q + 8 <= n; q += 8) {
+      for (; WIDE && q + 8 <= n; q += 8) {
         T av[8], bv[8];
 #pragma unroll
         for (int u = 0; u < 8; u++) { av[u] = a[(q + u) * sa]; bv[u] = b[(q + u) * sb]; }
@@ -771,7 +774,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         const int c = in.c, kk = in.k;
         RowCol rc(L.first(), c);
         for (int e = L.first(); e < w; e += es, rc.next(es, c)) {
-          const T s = dot(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk, neg_zero<T>());
+          const T s = dot<T, SHARED>(A.at(rc.i * kk), A.s, Bm.at(rc.j), c * Bm.s, kk, neg_zero<T>());
           L.st_mine(f[0], e, s);
           L.save_mine(f[3], e, s);
         }
@@ -990,7 +993,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
           RowCol rq(L.first(), kk);
           for (int e = L.first(); e < r * kk; e += es, rq.next(es, kk)) {
             T* q = L.wp(f[1]) + e * L.ss;
-            *q = dot(G_.at(rq.i * c), G_.s, Bm.at(rq.j * c), Bm.s, c, fa ? neg_zero<T>() : *q);
+            *q = dot<T, SHARED>(G_.at(rq.i * c), G_.s, Bm.at(rq.j * c), Bm.s, c, fa ? neg_zero<T>() : *q);
           }
         }
         if (f[2] != -1) {  // gB (k x c) += A^T (A is r x k) * gZ
@@ -998,7 +1001,7 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
           RowCol qj(L.first(), c);
           for (int e = L.first(); e < kk * c; e += es, qj.next(es, c)) {
             T* q = L.wp(f[2]) + e * L.ss;
-            *q = dot(A.at(qj.i), kk * A.s, G_.at(qj.j), c * G_.s, r, fb ? neg_zero<T>() : *q);
+            *q = dot<T, SHARED>(A.at(qj.i), kk * A.s, G_.at(qj.j), c * G_.s, r, fb ? neg_zero<T>() : *q);
           }
         }
         break;
@@ -1016,13 +1019,13 @@ __device__ __forceinline__ void replay_body(const ReplayArgs& a, const int block
         const uint32_t mn = div_magic(n);
         for (int e = L.first(); e < n * n; e += es) {
           const int p = divq(e, mn), j = e - p * n;
-          L.wp(f[2])[e * L.ss] = dot(G_.at(p * n), G_.s, Bv.at(j * n), Bv.s, n, neg_zero<T>());
+          L.wp(f[2])[e * L.ss] = dot<T, SHARED>(G_.at(p * n), G_.s, Bv.at(j * n), Bv.s, n, neg_zero<T>());
         }
         if (SHARED) __syncwarp();
         for (int e = L.first(); e < n * n; e += es) {
           const int i = divq(e, mn), j = e - i * n;
           T* q = L.wp(f[1]) + e * L.ss;
-          *q = -dot(Bv.at(i), n * Bv.s, M.at(j), n * M.s, n, fa ? neg_zero<T>() : -*q);
+          *q = -dot<T, SHARED>(Bv.at(i), n * Bv.s, M.at(j), n * M.s, n, fa ? neg_zero<T>() : -*q);
         }
         break;
       }
