@@ -16,7 +16,9 @@
 // coalesced run -- and copied back into slots ahead of use in the reverse sweep.
 //
 // GB300 note: FP64 issues at about 1/73 of the FP32 rate (one warp instruction per
-// 76 cycles per scheduler), and a dependent FP64 operation waits about 64 cycles.
+// 64 cycles per scheduler by the unit count, one per 76 in a saturated stream), and a
+// dependent FP64 operation waits about 64 cycles.  A warp instruction with lanes
+// predicated off still takes its full slot.
 // With enough warps the FP64 pipe binds; with few lanes (one warp per scheduler)
 // each lane's serial chain and the interpreter's own instructions set the time.
 // The cheap scalar rules therefore take a dispatch-free fused multiply-add path.
